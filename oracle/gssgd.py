@@ -1,0 +1,206 @@
+"""gs-SGD compression step, restated plainly on the CPU (test infrastructure only).
+
+One step for P data-parallel workers, in the order of Alg. 1 (Global Sketching SGD) and
+Alg. 2 (HEAVYMIX) of the paper:
+
+  1. accumulate   u_p <- rho*u_p + g_p ;  e_p <- e_p + u_p            (fp32 semantics)
+     Momentum and error feedback are named in Sec. II (1-bit SGD error feedback, DGC
+     momentum correction, and their being carried through a linear sketch); Alg. 1 itself
+     sketches the stochastic gradient directly.  The reading taken here keeps both
+     accumulators per worker and sketches the error accumulator e_p.
+  2. sketch       S_p = S(e_p), an r x c Count Sketch (Alg. 1 step 5, Sec. III-A)
+  3. tree merge   recursive halving over the P sketches (Alg. 1 steps 8-23; Sec. III-A for
+                  P not a power of two: with an odd number of participants the one with the
+                  largest id sits the round out)
+  4. query        est_i = median_j s_j(i) * S[j][h_j(i)]  (Alg. 2 step 1)
+  5. top-k        the k coordinates of largest |est|, ties to the smaller index
+                  (Alg. 2 steps 2-3 read as a deterministic top-k, see the design notes)
+  6. second round the exact values v_t = sum_p e_p[I_t] of the selected coordinates
+                  (Alg. 2 step 4), after which u_p and e_p are zeroed at I_t.
+
+Sketch cells, merge, median and gathered values are computed in fp64; alongside each table
+the oracle keeps the table of absolute contributions (sum of |s*x| per cell), which sets
+the tolerance bands used by the parity tests.
+"""
+
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+
+from .countsketch import hash_rows
+
+
+# ---- 1. accumulate ---------------------------------------------------------------------
+
+def _f32(x: np.ndarray) -> np.ndarray:
+    return np.asarray(x, dtype=np.float64).astype(np.float32)
+
+
+def accumulate(u: np.ndarray, e: np.ndarray, g: np.ndarray, rho: float):
+    """Return (u', e') with u' = fl(fl(rho*u) + g) and e' = fl(e + u'), fl = fp32 RN.
+
+    Each single operation is carried out in fp64 and rounded once to fp32; for one
+    +, - or * of fp32 operands this is exactly the IEEE fp32 round-to-nearest result.
+    No fused multiply-add is involved.  ``rho`` is taken as the fp32 value nearest to it.
+    """
+    rho32 = np.float64(np.float32(rho))
+    u64 = np.asarray(u, dtype=np.float32).astype(np.float64)
+    e64 = np.asarray(e, dtype=np.float32).astype(np.float64)
+    g64 = np.asarray(g, dtype=np.float32).astype(np.float64)
+    prod = _f32(rho32 * u64).astype(np.float64)
+    u_new = _f32(prod + g64)
+    e_new = _f32(e64 + u_new.astype(np.float64))
+    return u_new, e_new
+
+
+# ---- 2. sketch -------------------------------------------------------------------------
+
+def sketch(x: np.ndarray, coeffs, c: int):
+    """Count Sketch of vector x: (T, A), both [r, c] fp64.
+
+    T[j][b] = sum over i with h_j(i) = b of s_j(i) * x_i
+    A[j][b] = sum over the same i of |x_i|       (the magnitude carried by the cell)
+    """
+    x64 = np.asarray(x, dtype=np.float32).astype(np.float64)
+    d = x64.size
+    buckets, signs = hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+    r = buckets.shape[0]
+    T = np.zeros((r, c), dtype=np.float64)
+    A = np.zeros((r, c), dtype=np.float64)
+    ax = np.abs(x64)
+    for j in range(r):
+        T[j] = np.bincount(buckets[j], weights=signs[j] * x64, minlength=c)
+        A[j] = np.bincount(buckets[j], weights=ax, minlength=c)
+    return T, A
+
+
+# ---- 3. tree merge ---------------------------------------------------------------------
+
+def merge_schedule(P: int):
+    """Rounds of the recursive-halving reduce for P workers.
+
+    Round l (l = 0, 1, ...) involves the workers whose rank is a multiple of 2^l, listed
+    in rank order.  The participant at an even position receives from the next one and
+    adds; with an odd count the last (largest id) participant sits the round out.  The
+    result ends on worker 0 after ceil(log2 P) rounds.  Returns a list of rounds, each a
+    list of (receiver, sender) pairs.
+    """
+    rounds = []
+    step = 1
+    while step < P:
+        ranks = list(range(0, P, step))
+        pairs = [(ranks[m], ranks[m + 1]) for m in range(0, len(ranks) - 1, 2)]
+        rounds.append(pairs)
+        step *= 2
+    return rounds
+
+
+def merge_tree(tables):
+    """Sum the P tables along ``merge_schedule(P)``; returns the table left on worker 0.
+
+    ``tables`` is a list of arrays of equal shape; the inputs are not modified.
+    Each receive is 'sends = recvs + sends' (Alg. 1), done in fp64.
+    """
+    work = [np.array(t, dtype=np.float64, copy=True) for t in tables]
+    for pairs in merge_schedule(len(work)):
+        for recv, send in pairs:
+            work[recv] = work[send] + work[recv]
+    return work[0]
+
+
+# ---- 4. query --------------------------------------------------------------------------
+
+def query(T: np.ndarray, coeffs, d: int):
+    """est_i = median over rows j of s_j(i) * T[j][h_j(i)] for i < d (fp64).
+
+    With an odd number of rows the median is the middle order statistic; with an even
+    number it is the mean of the two middle ones.
+    """
+    c = T.shape[1]
+    buckets, signs = hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+    r = buckets.shape[0]
+    vals = np.empty((r, d), dtype=np.float64)
+    for j in range(r):
+        vals[j] = signs[j] * T[j][buckets[j]]
+    vals.sort(axis=0)
+    if r % 2 == 1:
+        return vals[r // 2].copy()
+    return 0.5 * (vals[r // 2 - 1] + vals[r // 2])
+
+
+def cell_band(A: np.ndarray, coeffs, idx, rel: float = 1e-5):
+    """Per-coordinate tolerance band rel * max_j A[j][h_j(i)] for the median estimate."""
+    c = A.shape[1]
+    buckets, _ = hash_rows(coeffs, c, np.asarray(idx, dtype=np.uint64))
+    r = buckets.shape[0]
+    mags = np.stack([A[j][buckets[j]] for j in range(r)])
+    return rel * mags.max(axis=0)
+
+
+# ---- 5. top-k --------------------------------------------------------------------------
+
+def topk(est: np.ndarray, k: int) -> np.ndarray:
+    """The k indices of largest |est|, ties broken toward the smaller index, ascending."""
+    est = np.asarray(est, dtype=np.float64)
+    order = np.lexsort((np.arange(est.size), -np.abs(est)))
+    return np.sort(order[:k]).astype(np.int64)
+
+
+# ---- 6. second round: gather exact values and zero the accumulators ---------------------
+
+def gather_and_zero(us, es, idx):
+    """Return (vals, us', es'): vals[t] = sum_p e_p[idx[t]] (fp64), accumulators zeroed.
+
+    The inputs are not modified.
+    """
+    idx = np.asarray(idx, dtype=np.int64)
+    vals = np.zeros(idx.size, dtype=np.float64)
+    for e in es:
+        vals += np.asarray(e, dtype=np.float32)[idx].astype(np.float64)
+    us_out, es_out = [], []
+    for u, e in zip(us, es):
+        u2 = np.array(u, dtype=np.float32, copy=True)
+        e2 = np.array(e, dtype=np.float32, copy=True)
+        u2[idx] = 0.0
+        e2[idx] = 0.0
+        us_out.append(u2)
+        es_out.append(e2)
+    return vals, us_out, es_out
+
+
+# ---- one full step ---------------------------------------------------------------------
+
+@dataclasses.dataclass
+class StepResult:
+    us: list            # per-worker momentum after the step (fp32)
+    es: list            # per-worker error accumulator after the step (fp32)
+    es_pre: list        # per-worker error accumulator after accumulate, before zeroing
+    tables: list        # per-worker sketch T_p (fp64 [r, c])
+    abs_tables: list    # per-worker magnitude tables A_p (fp64 [r, c])
+    merged: np.ndarray  # merged sketch (fp64 [r, c])
+    merged_abs: np.ndarray
+    est: np.ndarray     # fp64 [d]
+    idx: np.ndarray     # int64 [k], ascending
+    vals: np.ndarray    # fp64 [k]
+
+
+def step(us, es, gs, rho: float, coeffs, c: int, k: int) -> StepResult:
+    """One gs-SGD compression step over P workers (lists of fp32 vectors of length d)."""
+    P = len(gs)
+    d = np.asarray(gs[0]).size
+    us1, es1, tables, abs_tables = [], [], [], []
+    for p in range(P):
+        u1, e1 = accumulate(us[p], es[p], gs[p], rho)
+        T, A = sketch(e1, coeffs, c)
+        us1.append(u1)
+        es1.append(e1)
+        tables.append(T)
+        abs_tables.append(A)
+    merged = merge_tree(tables)
+    merged_abs = merge_tree(abs_tables)
+    est = query(merged, coeffs, d)
+    idx = topk(est, k)
+    vals, us2, es2 = gather_and_zero(us1, es1, idx)
+    return StepResult(us2, es2, es1, tables, abs_tables, merged, merged_abs, est, idx, vals)

@@ -1,0 +1,350 @@
+"""Pins of the CPU oracle against facts fixed outside the oracle itself.
+
+Each test checks the oracle against a published value, a closed form, an invariant of the
+Count Sketch (Sec. III-A: S(a) = C a is linear, so S(a + b) = S(a) + S(b)), the structure
+of the recursive-halving merge (Alg. 1 and the non-power-of-two rule of Sec. III-A), the
+output contract of Alg. 2 (exact values on the selected set, zero elsewhere), brute force
+on tiny inputs, or fp32 arithmetic as numpy performs it.  ``test_oracle_mutations`` plants
+plausible mistakes in copies of the oracle and checks that these pins catch them.
+"""
+
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import countsketch as cs
+from oracle import gssgd
+
+P61 = (1 << 61) - 1
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ---- coefficients ------------------------------------------------------------------------
+
+def test_splitmix64_published_vector():
+    lines = [l.strip() for l in open(os.path.join(GOLDEN, "splitmix64_seed1234567.txt"))
+             if l.strip() and not l.startswith("#")]
+    seed = int(lines[0].split()[1])
+    want = [int(x) for x in lines[1:]]
+    gen = oracle.splitmix64(seed)
+    assert [next(gen) for _ in want] == want
+
+
+def test_coefficients_ranges_and_order():
+    for seed in (0, 1, 42, 2**64 - 1):
+        a, b, a2, b2 = oracle.derive_coefficients(16, seed)
+        assert all(1 <= v <= P61 - 1 for v in a + a2)
+        assert all(0 <= v <= P61 - 1 for v in b + b2)
+    # four draws per row in the order a, b, a', b'
+    gen = oracle.splitmix64(7)
+    draws = [next(gen) for _ in range(8)]
+    a, b, a2, b2 = oracle.derive_coefficients(2, 7)
+    assert a[1] == 1 + draws[4] % (P61 - 1) and b2[0] == draws[3] % P61
+    assert oracle.derive_coefficients(3, 5) != oracle.derive_coefficients(3, 6)
+
+
+# ---- hash family -------------------------------------------------------------------------
+
+EXTREME_COEFFS = [
+    ([1], [0], [1], [0]),
+    ([P61 - 1], [P61 - 1], [P61 - 1], [P61 - 1]),
+    ([2**60 + 12345], [2**61 - 2], [3], [2**31 - 1]),
+    ([2**31 - 1], [2**31], [2**61 - 3], [1]),
+    ([(1 << 61) - (1 << 30)], [12345678901234567], [987654321987654], [P61 - 2]),
+]
+
+
+@pytest.mark.parametrize("c", [1, 2, 7, 1 << 14, 1000003, 1 << 26])
+def test_hash_numpy_matches_bigint(c):
+    rng = np.random.default_rng(c)
+    idx = np.concatenate([np.array([0, 1, 2, 3, 2**31 - 1, 2**31 - 2, 2**30, 11173961]),
+                          rng.integers(0, 2**31, 4000)]).astype(np.uint64)
+    coef_sets = EXTREME_COEFFS + [tuple(oracle.derive_coefficients(3, c))]
+    for co in coef_sets:
+        buckets, signs = oracle.hash_rows(co, c, idx)
+        for j in range(len(co[0])):
+            for t, i in enumerate(idx.tolist()):
+                assert buckets[j, t] == oracle.bucket_exact(co[0][j], co[1][j], c, i)
+                assert signs[j, t] == oracle.sign_exact(co[2][j], co[3][j], i)
+
+
+def test_hash_identity_and_negation_closed_forms():
+    i = np.arange(0, 2**31, 9973, dtype=np.uint64)
+    c = 1 << 20
+    # a = 1, b = 0: h(i) = i mod c; sign = parity of i
+    b1, s1 = oracle.hash_rows(([1], [0], [1], [0]), c, i)
+    assert np.array_equal(b1[0], (i % c).astype(np.int64))
+    assert np.array_equal(s1[0], np.where(i % 2 == 0, 1, -1))
+    # a = p - 1 = -1 (mod p), b = 0: h(i) = (p - i) mod c for i > 0
+    b2, _ = oracle.hash_rows(([P61 - 1], [0], [1], [0]), c, i[1:])
+    want = np.array([(P61 - int(v)) % c for v in i[1:]], dtype=np.int64)
+    assert np.array_equal(b2[0], want)
+
+
+def test_hash_rejects_large_coordinates():
+    with pytest.raises(ValueError):
+        oracle.hash_rows(([1], [0], [1], [0]), 8, np.array([2**31], dtype=np.uint64))
+
+
+# ---- accumulate --------------------------------------------------------------------------
+
+def test_accumulate_equals_numpy_fp32_arithmetic():
+    rng = np.random.default_rng(0)
+    n = 200_000
+    u = (rng.standard_normal(n) * 10.0 ** rng.integers(-30, 5, n)).astype(np.float32)
+    e = (rng.standard_normal(n) * 10.0 ** rng.integers(-30, 5, n)).astype(np.float32)
+    g = (rng.standard_normal(n) * 10.0 ** rng.integers(-30, 5, n)).astype(np.float32)
+    for rho in (0.9, 0.5, 0.0, 0.999):
+        u1, e1 = oracle.accumulate(u, e, g, rho)
+        r32 = np.float32(rho)
+        uw = (r32 * u) + g          # numpy float32 ops: one rounding each, never fused
+        ew = e + uw
+        assert uw.dtype == np.float32
+        assert np.array_equal(u1.view(np.uint32), uw.view(np.uint32))
+        assert np.array_equal(e1.view(np.uint32), ew.view(np.uint32))
+
+
+def test_accumulate_closed_form_dyadic():
+    # rho = 1/2, g = 1 every step, u_0 = e_0 = 0:
+    #   u_t = 2 - 2^(1-t),  e_t = 2t - 2 + 2^(1-t)   (exact in fp32 for small t)
+    u = np.zeros(3, np.float32)
+    e = np.zeros(3, np.float32)
+    g = np.ones(3, np.float32)
+    for t in range(1, 20):
+        u, e = oracle.accumulate(u, e, g, 0.5)
+        assert np.all(u == 2.0 - 2.0 ** (1 - t))
+        assert np.all(e == 2.0 * t - 2.0 + 2.0 ** (1 - t))
+
+
+# ---- sketch ------------------------------------------------------------------------------
+
+def _dyadic(rng, n, lo=-512, hi=512, scale=2.0**-10):
+    return (rng.integers(lo, hi, n) * scale).astype(np.float32)
+
+
+@pytest.mark.parametrize("r,c", [(1, 1), (3, 17), (5, 1 << 10), (7, 4096)])
+def test_sketch_linearity_exact(r, c):
+    rng = np.random.default_rng(r * c)
+    co = oracle.derive_coefficients(r, 99 + c)
+    x1, x2 = _dyadic(rng, 5000), _dyadic(rng, 5000)
+    T1, A1 = oracle.sketch(x1, co, c)
+    T2, _ = oracle.sketch(x2, co, c)
+    T12, _ = oracle.sketch(x1 + x2, co, c)   # x1 + x2 exact in fp32 for these values
+    assert np.array_equal(T1 + T2, T12)
+    Tm, _ = oracle.sketch(-3.0 * x1, co, c)  # homogeneity, exact for a power-of-two-ish 3
+    assert np.array_equal(Tm, -3.0 * T1)
+
+
+def test_sketch_row_sums_and_magnitudes():
+    rng = np.random.default_rng(3)
+    d, r, c = 3000, 5, 64
+    co = oracle.derive_coefficients(r, 3)
+    x = _dyadic(rng, d)
+    T, A = oracle.sketch(x, co, c)
+    for j in range(r):
+        want = sum(oracle.sign_exact(co[2][j], co[3][j], i) * float(x[i]) for i in range(d))
+        assert T[j].sum() == want
+        assert A[j].sum() == np.abs(x.astype(np.float64)).sum()
+        assert np.all(np.abs(T[j]) <= A[j])
+
+
+def test_single_spike_recovery():
+    d, r, c = 5000, 5, 1024
+    co = oracle.derive_coefficients(r, 11)
+    for i, v in ((0, 0.75), (1234, -3.5), (d - 1, 2.0**-20)):
+        x = np.zeros(d, np.float32)
+        x[i] = v
+        T, _ = oracle.sketch(x, co, c)
+        est = oracle.query(T, co, d)
+        assert est[i] == v
+        assert list(oracle.topk(est, 1)) == [i]
+        # every other coordinate sees v in at most some rows, so |est| <= |v|
+        assert np.all(np.abs(est) <= abs(v))
+
+
+def _injective_coeffs(r, seed):
+    """Rows with a = 1 and distinct offsets: h_j(i) = (i + b_j) mod c, injective for c >= d."""
+    rng = np.random.default_rng(seed)
+    a = [1] * r
+    b = [int(v) for v in rng.integers(0, 2**40, r)]
+    a2 = [int(v) for v in rng.integers(1, 2**60, r)]
+    b2 = [int(v) for v in rng.integers(0, 2**60, r)]
+    return a, b, a2, b2
+
+
+@pytest.mark.parametrize("r", [1, 3, 4, 5])
+def test_collision_free_sketch_is_exact(r):
+    rng = np.random.default_rng(r)
+    d = 700
+    co = _injective_coeffs(r, r)
+    x = rng.standard_normal(d).astype(np.float32)
+    x[::7] = x[1::7][: x[::7].size]            # plant exact ties of |x|
+    T, _ = oracle.sketch(x, co, c=d)
+    est = oracle.query(T, co, d)
+    assert np.array_equal(est, x.astype(np.float64))
+    for k in (1, 5, 100, d):
+        brute = sorted(range(d), key=lambda i: (-abs(float(x[i])), i))[:k]
+        assert list(oracle.topk(est, k)) == sorted(brute)
+
+
+@pytest.mark.parametrize("r", [3, 4, 5, 7])
+def test_median_ignores_one_contaminated_row(r):
+    # row 0: h(i) = 2i mod d, so i and i + d/2 share a bucket; other rows injective.
+    rng = np.random.default_rng(10 + r)
+    d = 512
+    a, b, a2, b2 = _injective_coeffs(r, 20 + r)
+    a[0], b[0] = 2, 0
+    co = (a, b, a2, b2)
+    x = rng.standard_normal(d).astype(np.float32)
+    T, _ = oracle.sketch(x, co, c=d)
+    est = oracle.query(T, co, d)
+    assert np.array_equal(est, x.astype(np.float64))
+
+
+def test_sketch_bruteforce_tiny():
+    rng = np.random.default_rng(5)
+    d, r, c = 40, 3, 7
+    co = oracle.derive_coefficients(r, 5)
+    x = rng.standard_normal(d).astype(np.float32)
+    T, A = oracle.sketch(x, co, c)
+    for j in range(r):
+        cells = [[] for _ in range(c)]
+        for i in range(d):
+            cells[oracle.bucket_exact(co[0][j], co[1][j], c, i)].append(
+                oracle.sign_exact(co[2][j], co[3][j], i) * float(x[i]))
+        for bkt in range(c):
+            assert math.isclose(T[j][bkt], math.fsum(cells[bkt]), rel_tol=1e-14, abs_tol=1e-14)
+            assert math.isclose(A[j][bkt], math.fsum(abs(v) for v in cells[bkt]),
+                                rel_tol=1e-14, abs_tol=1e-14)
+
+
+def test_count_sketch_error_bound():
+    """Accuracy sanity (not parity): with c buckets each row errs by about ||x||_2/sqrt(c);
+    by Chebyshev a row exceeds 3||x||_2/sqrt(c) with probability <= 1/9, and the median of
+    5 rows only when 3 rows do: probability <= 10/729 < 1.4 %."""
+    rng = np.random.default_rng(8)
+    d, r, c = 200_000, 5, 4096
+    co = oracle.derive_coefficients(r, 8)
+    x = (rng.standard_normal(d) * 1e-3).astype(np.float32)
+    heavy = rng.choice(d, 20, replace=False)
+    x[heavy] = np.float32(0.5)
+    T, _ = oracle.sketch(x, co, c)
+    est = oracle.query(T, co, d)
+    eps = 3.0 / math.sqrt(c)
+    err = np.abs(est - x.astype(np.float64))
+    assert np.mean(err > eps * np.linalg.norm(x.astype(np.float64))) < 10 / 729
+    assert set(oracle.topk(est, 20).tolist()) == set(heavy.tolist())
+
+
+# ---- merge -------------------------------------------------------------------------------
+
+def test_merge_schedule_structure():
+    S = oracle.merge_schedule
+    assert S(1) == []
+    assert S(2) == [[(0, 1)]]
+    assert S(4) == [[(0, 1), (2, 3)], [(0, 2)]]
+    assert S(5) == [[(0, 1), (2, 3)], [(0, 2)], [(0, 4)]]
+    assert S(6) == [[(0, 1), (2, 3), (4, 5)], [(0, 2)], [(0, 4)]]
+    for P in range(1, 70):
+        rounds = S(P)
+        assert len(rounds) == (0 if P == 1 else math.ceil(math.log2(P)))
+        sent, alive = set(), set(range(P))
+        for pairs in rounds:
+            involved = [q for pr in pairs for q in pr]
+            assert len(involved) == len(set(involved))          # one message per worker
+            for recv, send in pairs:
+                assert recv < send and recv in alive and send in alive
+                sent.add(send)
+                alive.discard(send)
+            # with an odd number of participants only the largest id sits out
+            step = 2 ** rounds.index(pairs)
+            parts = list(range(0, P, step))
+            idle = [q for q in parts if q not in involved]
+            assert idle == ([parts[-1]] if len(parts) % 2 else [])
+        assert alive == {0} and sent == set(range(1, P))
+
+
+@pytest.mark.parametrize("P", [1, 2, 3, 4, 5, 6, 7, 8, 9, 16, 32])
+def test_merge_equals_flat_sum_and_is_order_invariant(P):
+    rng = np.random.default_rng(P)
+    tabs = [(rng.integers(-2**20, 2**20, (3, 50)) * 2.0**-12) for _ in range(P)]
+    flat = np.sum(tabs, axis=0)
+    assert np.array_equal(oracle.merge_tree(tabs), flat)
+    perm = rng.permutation(P)
+    assert np.array_equal(oracle.merge_tree([tabs[q] for q in perm]), flat)
+
+
+def test_merge_of_sketches_is_sketch_of_sum():
+    rng = np.random.default_rng(12)
+    r, c, d, P = 5, 256, 4000, 6
+    co = oracle.derive_coefficients(r, 12)
+    xs = [_dyadic(rng, d, -64, 64, 2.0**-6) for _ in range(P)]
+    merged = oracle.merge_tree([oracle.sketch(x, co, c)[0] for x in xs])
+    total = np.sum(np.stack(xs).astype(np.float64), axis=0).astype(np.float32)
+    assert np.array_equal(merged, oracle.sketch(total, co, c)[0])
+
+
+# ---- top-k -------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("seed", range(6))
+def test_topk_bruteforce_with_ties(seed):
+    rng = np.random.default_rng(seed)
+    d = int(rng.integers(1, 65))
+    est = rng.choice(np.array([0.0, 1.0, -1.0, 2.5, -2.5, 0.25, 3.0]), d)
+    for k in range(1, d + 1):
+        brute = sorted(range(d), key=lambda i: (-abs(est[i]), i))[:k]
+        assert list(oracle.topk(est, k)) == sorted(brute)
+
+
+def test_topk_matches_stable_argsort():
+    rng = np.random.default_rng(4)
+    est = np.round(rng.standard_normal(100_000), 2)
+    k = 1234
+    ref = np.sort(np.argsort(-np.abs(est), kind="stable")[:k])
+    assert np.array_equal(oracle.topk(est, k), ref)
+
+
+# ---- second round ------------------------------------------------------------------------
+
+def test_gather_and_zero_conservation():
+    rng = np.random.default_rng(21)
+    d, P, k = 10_000, 8, 300
+    us = [_dyadic(rng, d) for _ in range(P)]
+    es = [_dyadic(rng, d) for _ in range(P)]
+    idx = np.sort(rng.choice(d, k, replace=False))
+    vals, us2, es2 = oracle.gather_and_zero(us, es, idx)
+    before = np.sum([e.astype(np.float64) for e in es], axis=0)
+    after = np.sum([e.astype(np.float64) for e in es2], axis=0)
+    full = after.copy()
+    full[idx] += vals
+    assert np.array_equal(full, before)
+    mask = np.ones(d, bool)
+    mask[idx] = False
+    for p in range(P):
+        assert np.all(us2[p][idx] == 0) and np.all(es2[p][idx] == 0)
+        assert np.array_equal(us2[p][mask].view(np.uint32), us[p][mask].view(np.uint32))
+        assert np.array_equal(es2[p][mask].view(np.uint32), es[p][mask].view(np.uint32))
+
+
+def test_step_output_contract():
+    """Alg. 2: exact (accumulated) values on the selected set, untouched accumulators
+    elsewhere; the selected set is the top-k of the estimate."""
+    rng = np.random.default_rng(31)
+    d, P, r, c, k = 5000, 4, 5, 512, 40
+    co = oracle.derive_coefficients(r, 31)
+    us = [np.zeros(d, np.float32) for _ in range(P)]
+    es = [np.zeros(d, np.float32) for _ in range(P)]
+    spikes = rng.choice(d, 10, replace=False)
+    for t in range(3):
+        gs = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        for g in gs:
+            g[spikes] += np.float32(0.1)
+        res = oracle.step(us, es, gs, 0.9, co, c, k)
+        assert np.array_equal(res.idx, oracle.topk(res.est, k))
+        assert set(spikes.tolist()) <= set(res.idx.tolist())
+        want = np.sum([e[res.idx].astype(np.float64) for e in res.es_pre], axis=0)
+        assert np.array_equal(res.vals, want)
+        us, es = res.us, res.es
