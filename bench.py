@@ -1,0 +1,407 @@
+"""Benchmark of the gs-SGD compression step on GB300.
+
+One step = the whole hot path for P simulated workers on one GPU: accumulate + Count
+Sketch insert (fused), tree merge, median query + top-k, gather-and-zero.  The metric is
+gradient coordinates per second, P * d * steps / time, for the ResNet-18-sized workload
+(d = 11,173,962, P = 8, r = 5, c = 2^17, k = 11,200) unless --config names another.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+Under torchrun (N > 1) every rank runs an independent replica of the workload on its own
+GPU (weak scaling, no collective on the data path); rank 0 prints one JSON line.
+--impl reference times the CPU oracle (the reference arm of this comparison) on bounded
+samples of the same workload.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import workloads  # noqa: E402
+
+METRIC = "gradient coords/s through accumulate+sketch+merge+top-k at P=8; % HBM roofline"
+UNIT = "coords/s"
+K1_SOURCE = os.path.join(ROOT, "paper_2108_06004_gb300", "csrc", "k_insert.cu")
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "accumulate_insert_resnet18.md")
+CPU_SAMPLE_D = 1 << 22   # coordinates per worker in one bounded oracle step (CPU baseline)
+REF_BUDGET_S = 120.0     # oracle seconds for a whole --impl reference run
+ORACLE_S_PER_COORD = 1.7e-7  # oracle seconds per worker-coordinate (sizes the reference samples)
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="resnet18", choices=sorted(workloads.CONFIGS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-steps", action="store_true",
+                    help="short run for a profiler: no e2e, no CPU baseline, no clocks")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+# ---- clocks ------------------------------------------------------------------------------
+
+class ClockSampler:
+    """nvidia-smi samples every 50 ms of the GPU (selected by UUID); stop() keeps the samples
+    whose own timestamps fall in the timed window (or, for a window shorter than the sampling
+    period, the samples nearest to it)."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu = gpu_id
+        self.proc = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-i", self.gpu,
+               "-lms", "50"]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.5)
+
+    def mark_begin(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+
+    def stop(self):
+        import datetime
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.2)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        inside = [x for x in rows if self.t0 <= x[0] <= self.t1]
+        if not inside and rows:
+            mid = 0.5 * (self.t0 + self.t1)
+            inside = sorted(rows, key=lambda x: abs(x[0] - mid))[:2]
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        reasons = sorted({n for x in inside for n, f in zip(self.NAMES, x[3]) if f.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(x[1] for x in inside), "sm_max_mhz": max(x[2] for x in inside),
+                "reasons": reasons, "samples": len(inside),
+                "window_s": round(self.t1 - self.t0, 3)}
+
+
+# ---- profile summary (ncu traffic) -------------------------------------------------------
+
+def k1_traffic_per_launch():
+    """DRAM bytes per launch of the fused accumulate+insert kernel from the committed ncu
+    summary, if that summary was taken on the current kernel source (else None)."""
+    try:
+        text = open(PROFILE_SUMMARY).read()
+    except OSError:
+        return None
+    src = hashlib.sha256(open(K1_SOURCE, "rb").read()).hexdigest()[:16]
+    m_sha = re.search(r"kernel source sha256\[:16\]:\s*`?([0-9a-f]{16})", text)
+    m_tr = re.search(r"traffic per full launch \(bytes\):\s*`?([0-9.eE+]+)", text)
+    if not m_sha or not m_tr or m_sha.group(1) != src:
+        return None
+    return float(m_tr.group(1))
+
+
+# ---- our arm -----------------------------------------------------------------------------
+
+def gpu_uuid(dev) -> str:
+    import torch
+    u = str(torch.cuda.get_device_properties(dev).uuid)
+    return u if u.startswith("GPU-") else "GPU-" + u
+
+
+def run_ours(args):
+    import torch
+    import paper_2108_06004_gb300 as gs
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    if not os.path.exists(gs.LIB_PATH):
+        if rank == 0 or world == 1:
+            from paper_2108_06004_gb300 import _build
+            _build.build()
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+    gs.load_library()
+
+    w = workloads.get_config(args.config)
+    P, d, r, c, k, rho = w.P, w.d, w.r, w.c, w.k, w.rho
+    nsteps_pool = min(w.steps, max(1, args.steps + args.warmup))
+    # Fresh gradients for each of the workload's steps (cycled if more steps are timed).
+    # Replicas on different ranks draw different workers' gradients.
+    host_pool = []
+    for t in range(nsteps_pool):
+        gl = workloads.make_gradients(w, t, [rank * P + p for p in range(P)])
+        host_pool.append([torch.from_numpy(g).pin_memory() for g in gl])
+    dev_pool = [[g.to(dev, non_blocking=True) for g in step] for step in host_pool]
+    us = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
+    es = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
+    sk = gs.gs_sketch_create(r, c, 20210813, P, 0)
+    W = gs.gs_sketch_info(sk)["group_width"]
+    groups = (P + W - 1) // W
+    ws = torch.empty(gs.gs_step_workspace_size(d, k), dtype=torch.uint8, device=dev)
+    qws_bytes = gs.gs_query_topk_workspace_size(d, k)
+    idx = torch.empty(k, dtype=torch.int64, device=dev)
+    vals = torch.empty(k, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+
+    k1_events = []
+
+    def step(t, record):
+        grads = dev_pool[t % nsteps_pool]
+        gs.gs_sketch_zero(sk, stream)
+        for g0 in range(0, P, W):
+            if record:
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            gs.gs_accumulate_insert(sk, g0, us[g0:g0 + W], es[g0:g0 + W], grads[g0:g0 + W], d, rho, stream)
+            if record:
+                e1.record(stream)
+                k1_events.append((e0, e1, min(W, P - g0)))
+        gs.gs_sketch_merge_tree(sk, P, stream)
+        gs.gs_query_topk(sk, d, k, idx, None, ws, qws_bytes, stream)
+        gs.gs_gather_and_zero(us, es, d, idx, k, vals, stream)
+
+    for t in range(args.warmup):
+        step(t, False)
+    torch.cuda.synchronize()
+
+    clocks = None
+    sampler = None
+    if not args.profile_steps:
+        sampler = ClockSampler(gpu_uuid(dev))
+        sampler.start()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark_begin()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for t in range(args.steps):
+        step(args.warmup + t, True)
+    end.record(stream)
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark_end()
+    elapsed_ms = start.elapsed_time(end)
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        dist.barrier()
+        elapsed_ms = float(tt.item())
+    if sampler:
+        clocks = sampler.stop()
+
+    k1_ms = [a.elapsed_time(b) for a, b, _ in k1_events]
+    k1_lanes = [n for _, _, n in k1_events]
+    coords = world * P * d * args.steps
+    value = coords / (elapsed_ms / 1e3)
+
+    # roofline of the dominant kernel: fused accumulate + insert (20 algorithmic HBM bytes per
+    # worker-coordinate: read g, u, e; write u, e)
+    peaks, peak_kind = measured_peaks()
+    k1_bytes = [20.0 * n * d for n in k1_lanes]
+    k1_avg_s = (sum(k1_ms) / len(k1_ms)) / 1e3
+    k1_gbs = (sum(k1_bytes) / len(k1_bytes)) / k1_avg_s / 1e9
+    full_launch_bytes = 20.0 * W * d
+    reds_per_launch = d * r * ((W + 3) // 4)
+    roofline = {
+        "kernel": "k_accumulate_insert (fused S1+S2)",
+        "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+        "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
+        "traffic": k1_traffic_per_launch(),
+        "algorithmic_bytes_per_launch": full_launch_bytes,
+        "avg_launch_ms": round(sum(k1_ms) / len(k1_ms), 4),
+        "co_bound": {"kind": "l2_vector_reductions", "per_launch": reds_per_launch,
+                     "achieved_G_per_s": round(reds_per_launch / k1_avg_s / 1e9, 1),
+                     "probe_peak_G_per_s": 195.0},
+        "step_share": round(sum(k1_ms) / elapsed_ms, 3),
+    }
+
+    # end to end through the public call with host buffers
+    e2e = None
+    if not args.no_e2e and not args.profile_steps:
+        grad_dev = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(P)]
+        idx_h = torch.empty(k, dtype=torch.int64).pin_memory()
+        vals_h = torch.empty(k, dtype=torch.float32).pin_memory()
+        for t in range(args.warmup):
+            gs.gs_step_host(sk, us, es, host_pool[t % nsteps_pool], grad_dev, d, rho, k, idx_h, vals_h, ws,
+                            None, stream)
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for t in range(args.steps):
+            gs.gs_step_host(sk, us, es, host_pool[(args.warmup + t) % nsteps_pool], grad_dev, d, rho, k, idx_h,
+                            vals_h, ws, None, stream)
+        torch.cuda.synchronize()
+        e2e_s = time.perf_counter() - t0
+        if world > 1:
+            import torch.distributed as dist
+            tt = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e2e_s = float(tt.item())
+        e2e = {"value": coords / e2e_s, "unit": UNIT, "h2d_bytes_per_step": P * d * 4,
+               "d2h_bytes_per_step": k * (8 + 4), "ms_per_step": round(e2e_s * 1e3 / args.steps, 4),
+               "call": "gs_step_host"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_steps:
+        cpu = cpu_baseline(w, steps=2)
+
+    gs.gs_sketch_destroy(sk)
+    launches_per_step = groups + 1 + 9 + 1  # insert groups, merge, query/top-k (9), gather
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": w.name, "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
+                   "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
+                   "l2": f"inputs larger than L2 ({P * d * 12 / 1e9:.2f} GB of g,u,e streamed per step)",
+                   "d_steps_per_s": world * d * args.steps / (elapsed_ms / 1e3)},
+        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+# ---- the CPU oracle as baseline / reference arm -------------------------------------------
+
+def _oracle_sample_step(w, t, d_s, k_s, coeffs, us, es):
+    import oracle
+    grads = workloads.make_gradients(w, t, range(w.P), d=d_s)
+    t0 = time.perf_counter()
+    res = oracle.step(us, es, grads, w.rho, coeffs, w.c, k_s)
+    dt = time.perf_counter() - t0
+    return dt, res
+
+
+def cpu_baseline(w, steps=1, d_s=CPU_SAMPLE_D):
+    """The oracle, as it stands, on the first d_s coordinates of each worker's gradient
+    (same P, r, c and rho; k scaled with d); the same unit as the metric."""
+    import oracle
+    k_s = max(1, round(w.k * d_s / w.d))
+    coeffs = oracle.derive_coefficients(w.r, 20210813)
+    us = [np.zeros(d_s, np.float32) for _ in range(w.P)]
+    es = [np.zeros(d_s, np.float32) for _ in range(w.P)]
+    total = 0.0
+    for t in range(steps):
+        dt, res = _oracle_sample_step(w, t, d_s, k_s, coeffs, us, es)
+        total += dt
+        us, es = res.us, res.es
+    return {"value": w.P * d_s * steps / total, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{steps} step(s) of the oracle on the first {d_s} coordinates of each of the {w.P} "
+                      f"workers (r={w.r}, c={w.c}, k={k_s}), numpy single-threaded"}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    import oracle
+    w = workloads.get_config(args.config)
+    per_step = REF_BUDGET_S / max(1, args.steps + args.warmup)
+    d_s = 1 << 16
+    while d_s * 2 <= min(w.d, 1 << 22) and 2 * d_s * w.P * ORACLE_S_PER_COORD <= per_step:
+        d_s *= 2
+    k_s = max(1, round(w.k * d_s / w.d))
+    coeffs = oracle.derive_coefficients(w.r, 20210813)
+    us = [np.zeros(d_s, np.float32) for _ in range(w.P)]
+    es = [np.zeros(d_s, np.float32) for _ in range(w.P)]
+    for t in range(args.warmup):
+        _, res = _oracle_sample_step(w, t, d_s, k_s, coeffs, us, es)
+        us, es = res.us, res.es
+    total = 0.0
+    for t in range(args.steps):
+        dt, res = _oracle_sample_step(w, args.warmup + t, d_s, k_s, coeffs, us, es)
+        total += dt
+        us, es = res.us, res.es
+    value = w.P * d_s * args.steps / total
+    sample = (f"each step: the oracle on the first {d_s} coordinates of each of the {w.P} workers "
+              f"(r={w.r}, c={w.c}, k={k_s}), numpy single-threaded")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total * 1e3 / args.steps, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "d": w.d, "P": w.P, "r": w.r, "c": w.c, "k": w.k, "rho": w.rho},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

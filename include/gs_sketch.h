@@ -1,0 +1,197 @@
+/*
+ * gs_sketch.h -- C ABI of the GB300 gs-SGD gradient-compression library.
+ *
+ * The library runs the per-step compression pipeline of global-sketching SGD
+ * (Dai, Diao, Li, Xu, arXiv 2108.06004) for P data-parallel workers simulated on one
+ * GPU:
+ *
+ *   accumulate    u_p <- rho*u_p + g_p,  e_p <- e_p + u_p       (momentum + error feedback)
+ *   insert        T_p <- T_p + S(e_p), an r x c Count Sketch     (Alg. 1 step 5, Sec. III-A)
+ *   merge         recursive-halving tree of the P sketches       (Alg. 1 steps 8-23)
+ *   query + top-k est_i = median_j s_j(i) T[j][h_j(i)], top-k of |est|  (Alg. 2 steps 1-3)
+ *   gather + zero v_t = sum_p e_p[I_t]; u_p[I_t] = e_p[I_t] = 0  (Alg. 2 step 4)
+ *
+ * Hash family (the paper names Count Sketch but prints no family): for row j,
+ *   h_j(i) = ((a_j*i + b_j) mod (2^61 - 1)) mod c,
+ *   s_j(i) = +1 if ((a'_j*i + b'_j) mod (2^61 - 1)) is even, else -1,
+ * with (a_j, b_j, a'_j, b'_j) the next four outputs of splitmix64(seed) (Steele, Lea and
+ * Flood, OOPSLA 2014) reduced as a = 1 + x mod (2^61 - 2), b = x mod (2^61 - 1).
+ *
+ * Conventions for every call
+ *   - Vectors, index and value arrays and workspaces are CALLER-OWNED DEVICE pointers
+ *     unless a parameter says "host".  The library owns only sketch tables.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy default
+ *     stream) except those documented as synchronous.  The current CUDA device must be
+ *     the device the sketch was created on.
+ *   - Arguments are validated on the host before any launch; a failed check returns
+ *     GS_ERR_INVALID_ARG (or GS_ERR_MISMATCH) and launches nothing.  A CUDA error
+ *     returns GS_ERR_CUDA.  gs_last_error() then gives a message (thread-local).
+ *   - fp32 vectors must be 4-byte aligned; 16-byte alignment of every vector selects
+ *     the vectorised path (results are identical either way).
+ *   - Sizes: 1 <= r <= GS_MAX_ROWS, 1 <= c <= GS_MAX_COLS, 1 <= d <= GS_MAX_DIM,
+ *     1 <= k <= d, 1 <= P <= GS_MAX_WORKERS.  Vector values must be finite.
+ *   - No call waits on the device for a flag; nothing spins.
+ */
+#ifndef GS_SKETCH_H
+#define GS_SKETCH_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t gs_status;
+#define GS_OK 0
+#define GS_ERR_INVALID_ARG 1
+#define GS_ERR_MISMATCH 2
+#define GS_ERR_OOM 3
+#define GS_ERR_CUDA 4
+#define GS_ERR_TIMEOUT 5
+
+#define GS_MAX_ROWS 16
+#define GS_MAX_COLS (1 << 26)
+#define GS_MAX_WORKERS 64
+#define GS_MAX_DIM 2147483647LL /* d < 2^31 */
+
+typedef struct gs_sketch gs_sketch; /* opaque */
+typedef void* gs_stream;            /* a cudaStream_t */
+
+/* ---- sketch lifetime ------------------------------------------------------------- */
+
+/* Create a set of `workers` Count Sketches of r rows x c columns sharing one hash family
+ * drawn from `seed` (Sec. III-A: sketches combine by addition only when they share their
+ * hash functions), plus the merged r x c table that gs_sketch_merge_tree writes.
+ * All tables start at zero.  Worker tables are stored interleaved in groups of
+ * `group_width` workers ([group][r][c][group_width] fp32) so that one 16-byte vector
+ * reduction updates four workers' cells at once; group_width 0 lets the library choose
+ * (the widest of 8, 4, 2, 1 whose group table fits a fixed L2-sized budget).
+ * On success *out owns device memory released by gs_sketch_destroy.
+ * Errors: GS_ERR_INVALID_ARG (sizes, group_width not in {0,1,2,4,8}, out NULL),
+ *         GS_ERR_OOM (allocation failed), GS_ERR_CUDA.  Synchronous. */
+gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
+                           int32_t group_width, gs_sketch** out);
+
+/* Release a sketch and its device memory.  NULL is accepted.  Synchronous. */
+gs_status gs_sketch_destroy(gs_sketch* sketch);
+
+/* Shape query: any output pointer may be NULL. */
+gs_status gs_sketch_info(const gs_sketch* sketch, int32_t* r, int32_t* c, int32_t* workers,
+                         int32_t* group_width);
+
+/* Host copy of the hash coefficients: out4r[4*j + {0,1,2,3}] = a_j, b_j, a'_j, b'_j
+ * (host array of 4*r uint64).  Synchronous, no device work. */
+gs_status gs_sketch_coefficients(const gs_sketch* sketch, uint64_t* out4r);
+
+/* Zero every worker table and the merged table (start of a step). */
+gs_status gs_sketch_zero(gs_sketch* sketch, gs_stream stream);
+
+/* ---- step 1: accumulate ---------------------------------------------------------- */
+
+/* u <- fl(fl(rho*u) + g); e <- fl(e + u) elementwise over d fp32 values, each operation
+ * rounded to nearest in fp32 and never fused (momentum correction and error feedback,
+ * Sec. II).  momentum and error are updated in place; grad is read only.  The three
+ * arrays must not overlap. */
+gs_status gs_accumulate(float* momentum, float* error, const float* grad, int64_t d,
+                        float rho, gs_stream stream);
+
+/* ---- step 2: sketch insert ------------------------------------------------------- */
+
+/* T_worker[j][h_j(i)] += s_j(i) * vec[i] for all rows j and i < d (Alg. 1 step 5).
+ * Cells are fp32 and updated with atomic additions, so their rounding order is not
+ * fixed.  0 <= worker < workers. */
+gs_status gs_sketch_insert(gs_sketch* sketch, int32_t worker, const float* vec, int64_t d,
+                           gs_stream stream);
+
+/* Fused steps 1+2 for workers first_worker .. first_worker+n_workers-1: for each such
+ * worker p (array entry p - first_worker), gs_accumulate on (momentum, error, grad) and
+ * then insert the updated error vector into T_p, in one pass over the vectors.  The
+ * pointer arrays are HOST arrays of n_workers DEVICE pointers.  first_worker must be a
+ * multiple of the group width, and the range must end on a group boundary or at the
+ * last worker.  Per worker the result equals gs_accumulate followed by gs_sketch_insert
+ * (up to the order of the fp32 atomic additions in the cells). */
+gs_status gs_accumulate_insert(gs_sketch* sketch, int32_t first_worker, int32_t n_workers,
+                               float* const* momentum, float* const* error,
+                               const float* const* grad, int64_t d, float rho,
+                               gs_stream stream);
+
+/* ---- step 3: tree merge ---------------------------------------------------------- */
+
+/* Merge the tables of workers 0..P-1 into the merged table by recursive halving
+ * (Alg. 1 steps 8-23): in round l the workers whose rank is a multiple of 2^l take part
+ * in rank order; each one at an even position adds the table of the next one to its own
+ * ("sends = recvs + sends"); with an odd number of participants the largest rank sits the
+ * round out (Sec. III-A).  ceil(log2 P) rounds; the fp32 additions follow exactly this
+ * order for every cell.  Worker tables are left unchanged. */
+gs_status gs_sketch_merge_tree(gs_sketch* sketch, int32_t P, gs_stream stream);
+
+/* ---- steps 4-5: median query and top-k ------------------------------------------- */
+
+/* Device workspace bytes gs_query_topk needs for d coordinates and k selected. */
+gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes);
+
+/* From the merged table: est_i = median over rows j of s_j(i) * T[j][h_j(i)] (fp32; the
+ * middle value for odd r, the mean of the two middle values for even r), then the k
+ * coordinates of largest |est_i|, ties toward the smaller index, written to idx_out
+ * (int64[k]) in ascending order (Alg. 2 steps 1-3).  est_out (fp32[d]) may be NULL.
+ * workspace must hold gs_query_topk_workspace_size(d, k) bytes, 256-byte aligned. */
+gs_status gs_query_topk(const gs_sketch* sketch, int64_t d, int64_t k, int64_t* idx_out,
+                        float* est_out, void* workspace, size_t workspace_bytes,
+                        gs_stream stream);
+
+/* ---- step 6: second round -------------------------------------------------------- */
+
+/* vals_out[t] = sum over p = 0..P-1 (in that order, fp32) of error[p][idx[t]], then
+ * momentum[p][idx[t]] = error[p][idx[t]] = 0 for every p (Alg. 2 step 4).  momentum and
+ * error are HOST arrays of P DEVICE pointers.  idx holds k distinct indices in [0, d);
+ * an index outside that range is skipped (no memory is touched) and its value is NaN. */
+gs_status gs_gather_and_zero(float* const* momentum, float* const* error, int32_t P,
+                             int64_t d, const int64_t* idx, int64_t k, float* vals_out,
+                             gs_stream stream);
+
+/* ---- whole step ------------------------------------------------------------------ */
+
+/* Device workspace bytes gs_step needs (query workspace plus the step's own buffers). */
+gs_status gs_step_workspace_size(int64_t d, int64_t k, size_t* bytes);
+
+/* One full compression step for workers 0..P-1 (P = the sketch's worker count):
+ * gs_sketch_zero, gs_accumulate_insert over all groups, gs_sketch_merge_tree(P),
+ * gs_query_topk, gs_gather_and_zero -- all on `stream`, asynchronous.  All pointers are
+ * device pointers (pointer arrays are host arrays of P device pointers); est_out may be
+ * NULL. */
+gs_status gs_step(gs_sketch* sketch, float* const* momentum, float* const* error,
+                  const float* const* grad, int64_t d, float rho, int64_t k,
+                  int64_t* idx_out, float* vals_out, float* est_out, void* workspace,
+                  size_t workspace_bytes, gs_stream stream);
+
+/* gs_step with the gradients in HOST memory and the results returned to HOST memory:
+ * copies grad_host[p] (pinned host memory gives full copy speed) into the device buffers
+ * grad_dev[p], runs gs_step, copies idx (int64[k]) and vals (fp32[k]) back to idx_host
+ * and vals_host, and synchronizes `stream` before returning.  Momentum and error stay
+ * resident on the device. */
+gs_status gs_step_host(gs_sketch* sketch, float* const* momentum, float* const* error,
+                       const float* const* grad_host, float* const* grad_dev, int64_t d,
+                       float rho, int64_t k, int64_t* idx_host, float* vals_host,
+                       void* workspace, size_t workspace_bytes, gs_stream stream);
+
+/* ---- inspection hooks ------------------------------------------------------------ */
+
+/* Buckets and signs of n coordinates for every row: bucket_out[j*n + t] = h_j(coords[t]),
+ * sign_out[j*n + t] = s_j(coords[t]) (int32 / int8 device arrays of r*n).  Coordinates
+ * must lie in [0, 2^31); others give bucket -1 and sign 0. */
+gs_status gs_hash_eval(const gs_sketch* sketch, const int64_t* coords, int64_t n,
+                       int32_t* bucket_out, int8_t* sign_out, gs_stream stream);
+
+/* Copy one table to HOST memory host_out (fp32 [r][c]): worker >= 0 gives that worker's
+ * table, worker == -1 the merged table.  Synchronous (waits for all prior device work). */
+gs_status gs_sketch_copy_to_host(const gs_sketch* sketch, int32_t worker, float* host_out);
+
+/* Message for the last non-OK status returned on this thread ("" if none). */
+const char* gs_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GS_SKETCH_H */

@@ -57,15 +57,16 @@ def accumulate(u: np.ndarray, e: np.ndarray, g: np.ndarray, rho: float):
 
 # ---- 2. sketch -------------------------------------------------------------------------
 
-def sketch(x: np.ndarray, coeffs, c: int):
+def sketch(x: np.ndarray, coeffs, c: int, hashes=None):
     """Count Sketch of vector x: (T, A), both [r, c] fp64.
 
     T[j][b] = sum over i with h_j(i) = b of s_j(i) * x_i
     A[j][b] = sum over the same i of |x_i|       (the magnitude carried by the cell)
+    ``hashes`` may pass ``hash_rows(coeffs, c, arange(d))`` computed once for many vectors.
     """
     x64 = np.asarray(x, dtype=np.float32).astype(np.float64)
     d = x64.size
-    buckets, signs = hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+    buckets, signs = hashes if hashes is not None else hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
     r = buckets.shape[0]
     T = np.zeros((r, c), dtype=np.float64)
     A = np.zeros((r, c), dtype=np.float64)
@@ -112,14 +113,14 @@ def merge_tree(tables):
 
 # ---- 4. query --------------------------------------------------------------------------
 
-def query(T: np.ndarray, coeffs, d: int):
+def query(T: np.ndarray, coeffs, d: int, hashes=None):
     """est_i = median over rows j of s_j(i) * T[j][h_j(i)] for i < d (fp64).
 
     With an odd number of rows the median is the middle order statistic; with an even
     number it is the mean of the two middle ones.
     """
     c = T.shape[1]
-    buckets, signs = hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+    buckets, signs = hashes if hashes is not None else hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
     r = buckets.shape[0]
     vals = np.empty((r, d), dtype=np.float64)
     for j in range(r):
@@ -176,6 +177,7 @@ def gather_and_zero(us, es, idx):
 class StepResult:
     us: list            # per-worker momentum after the step (fp32)
     es: list            # per-worker error accumulator after the step (fp32)
+    us_pre: list        # per-worker momentum after accumulate, before zeroing
     es_pre: list        # per-worker error accumulator after accumulate, before zeroing
     tables: list        # per-worker sketch T_p (fp64 [r, c])
     abs_tables: list    # per-worker magnitude tables A_p (fp64 [r, c])
@@ -190,17 +192,18 @@ def step(us, es, gs, rho: float, coeffs, c: int, k: int) -> StepResult:
     """One gs-SGD compression step over P workers (lists of fp32 vectors of length d)."""
     P = len(gs)
     d = np.asarray(gs[0]).size
+    hashes = hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))  # shared by all workers
     us1, es1, tables, abs_tables = [], [], [], []
     for p in range(P):
         u1, e1 = accumulate(us[p], es[p], gs[p], rho)
-        T, A = sketch(e1, coeffs, c)
+        T, A = sketch(e1, coeffs, c, hashes)
         us1.append(u1)
         es1.append(e1)
         tables.append(T)
         abs_tables.append(A)
     merged = merge_tree(tables)
     merged_abs = merge_tree(abs_tables)
-    est = query(merged, coeffs, d)
+    est = query(merged, coeffs, d, hashes)
     idx = topk(est, k)
     vals, us2, es2 = gather_and_zero(us1, es1, idx)
-    return StepResult(us2, es2, es1, tables, abs_tables, merged, merged_abs, est, idx, vals)
+    return StepResult(us2, es2, us1, es1, tables, abs_tables, merged, merged_abs, est, idx, vals)

@@ -1,0 +1,78 @@
+"""Compile the CUDA library libgs_sketch.so for sm_103a with nvcc, in-tree.
+
+Each translation unit is compiled in parallel to an object under ``_build/`` and the
+objects are linked into ``libgs_sketch.so`` next to this file.  The CUDA runtime is linked
+dynamically (soname libcudart.so.13), so inside a PyTorch process the library shares
+PyTorch's runtime instance and its current device and context.
+"""
+
+from __future__ import annotations
+
+import os
+import shutil
+import subprocess
+from concurrent.futures import ThreadPoolExecutor
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(HERE)
+CSRC = os.path.join(HERE, "csrc")
+INCLUDE = os.path.join(ROOT, "include")
+BUILD_DIR = os.path.join(HERE, "_build")
+LIB_PATH = os.path.join(HERE, "libgs_sketch.so")
+SOURCES = ["gs_api.cu", "k_insert.cu", "k_merge.cu", "k_query_topk.cu", "k_gather.cu"]
+ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+CFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xptxas", "-v",
+                 "-I", INCLUDE, "-I", CSRC]
+
+
+def _nvcc() -> str:
+    path = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
+    if not os.path.exists(path):
+        raise RuntimeError("nvcc not found: the CUDA toolkit is required to build libgs_sketch.so")
+    return path
+
+
+def _cuda_libdir(nvcc: str) -> str:
+    root = os.path.dirname(os.path.dirname(os.path.realpath(nvcc)))
+    for cand in ("lib64", "lib"):
+        d = os.path.join(root, cand)
+        if os.path.isdir(d):
+            return d
+    return os.path.join(root, "lib64")
+
+
+def _compile(nvcc: str, src: str) -> str:
+    obj = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + ".o")
+    log = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + ".ptxas.log")
+    cmd = [nvcc, *CFLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
+    res = subprocess.run(cmd, capture_output=True, text=True)
+    with open(log, "w") as f:
+        f.write(res.stdout + res.stderr)
+    if res.returncode != 0:
+        raise RuntimeError(f"nvcc failed on {src}:\n{res.stderr[-4000:]}")
+    return obj
+
+
+def build(verbose: bool = False) -> str:
+    """Compile every translation unit and link the shared library; returns its path."""
+    nvcc = _nvcc()
+    os.makedirs(BUILD_DIR, exist_ok=True)
+    with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
+        objs = list(ex.map(lambda s: _compile(nvcc, s), SOURCES))
+    libdir = _cuda_libdir(nvcc)
+    tmp = LIB_PATH + ".tmp"
+    cmd = [nvcc, *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs,
+           "-Xlinker", f"-rpath,{libdir}"]
+    res = subprocess.run(cmd, capture_output=True, text=True)
+    if res.returncode != 0:
+        raise RuntimeError(f"link failed:\n{res.stderr[-4000:]}")
+    os.replace(tmp, LIB_PATH)
+    if verbose:
+        for s in SOURCES:
+            print(open(os.path.join(BUILD_DIR, os.path.splitext(s)[0] + ".ptxas.log")).read())
+    return LIB_PATH
+
+
+if __name__ == "__main__":
+    import sys
+    print(build(verbose="-v" in sys.argv))

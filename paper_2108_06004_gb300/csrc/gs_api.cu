@@ -1,0 +1,525 @@
+// C ABI of the gs-SGD compression library: argument validation, the sketch object, hash
+// coefficient derivation, and composition of the kernels into the calls of gs_sketch.h.
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+#include <unordered_map>
+#include <vector>
+
+#include "gs_common.cuh"
+
+struct gs_sketch {
+  int32_t r, c, workers, W, groups;
+  uint64_t seed;
+  gs::HashCoeffs h;
+  float* tables;  // groups * r*c*W
+  float* merged;  // r*c
+  int device;
+};
+
+namespace {
+
+thread_local std::string g_err;
+
+gs_status fail(gs_status st, const std::string& msg) {
+  g_err = msg;
+  return st;
+}
+
+gs_status cuda_fail(cudaError_t e, const char* what) {
+  g_err = std::string(what) + ": " + cudaGetErrorString(e);
+  return GS_ERR_CUDA;
+}
+
+gs_status ok() {
+  return GS_OK;
+}
+
+// splitmix64 (Steele, Lea and Flood, OOPSLA 2014): advance the state by the golden-ratio
+// increment and mix it with two xor-shift-multiply rounds.
+uint64_t splitmix64_next(uint64_t& state) {
+  state += 0x9E3779B97F4A7C15ull;
+  uint64_t z = state;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+void derive_coefficients(int r, uint64_t seed, gs::HashCoeffs& h) {
+  std::memset(&h, 0, sizeof(h));
+  uint64_t state = seed;
+  for (int j = 0; j < r; ++j) {
+    h.a[j] = 1 + splitmix64_next(state) % (gs::kP61 - 1);
+    h.b[j] = splitmix64_next(state) % gs::kP61;
+    h.a2[j] = 1 + splitmix64_next(state) % (gs::kP61 - 1);
+    h.b2[j] = splitmix64_next(state) % gs::kP61;
+  }
+}
+
+constexpr size_t kGroupBudgetBytes = size_t(64) << 20;  // interleaved group table kept L2-sized
+
+int choose_group_width(int r, int c, int workers) {
+  int cap = 1;
+  while (cap < workers && cap < gs::kMaxGroup) cap *= 2;
+  for (int W = cap; W > 1; W /= 2) {
+    if ((size_t)r * (size_t)c * (size_t)W * sizeof(float) <= kGroupBudgetBytes) return W;
+  }
+  return 1;
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+gs_status check_sketch(const gs_sketch* sk) {
+  if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev != sk->device)
+    return fail(GS_ERR_INVALID_ARG, "current device " + std::to_string(dev) +
+                                        " differs from the sketch's device " + std::to_string(sk->device));
+  return GS_OK;
+}
+
+gs_status check_d(int64_t d) {
+  if (d < 1 || d > GS_MAX_DIM) return fail(GS_ERR_INVALID_ARG, "d must lie in [1, 2^31 - 1], got " + std::to_string(d));
+  return GS_OK;
+}
+
+gs_status check_vec(const void* p, const char* name) {
+  if (!p) return fail(GS_ERR_INVALID_ARG, std::string(name) + " is NULL");
+  if (!aligned(p, 4)) return fail(GS_ERR_INVALID_ARG, std::string(name) + " is not 4-byte aligned");
+  return GS_OK;
+}
+
+#define GS_TRY(expr)                  \
+  do {                                \
+    const gs_status st__ = (expr);    \
+    if (st__ != GS_OK) return st__;   \
+  } while (0)
+
+#define GS_GUARD_BEGIN try {
+#define GS_GUARD_END                                                  \
+  }                                                                   \
+  catch (const std::bad_alloc&) {                                     \
+    return fail(GS_ERR_OOM, "host allocation failed");                \
+  }                                                                   \
+  catch (...) {                                                       \
+    return fail(GS_ERR_INVALID_ARG, "unexpected host exception");     \
+  }
+
+cudaStream_t as_stream(gs_stream s) { return reinterpret_cast<cudaStream_t>(s); }
+
+gs_status accumulate_insert_impl(gs_sketch* sk, int32_t first, int32_t n, float* const* m,
+                                 float* const* e, const float* const* g, int64_t d, float rho,
+                                 cudaStream_t s) {
+  const int W = sk->W;
+  const int end = first + n;
+  for (int grp = first / W; grp * W < end; ++grp) {
+    gs::InsertParams p;
+    std::memset(&p, 0, sizeof(p));
+    const int lo = grp * W;
+    const int nw = (end - lo) < W ? (end - lo) : W;
+    bool vec = true;
+    for (int w = 0; w < nw; ++w) {
+      const int a = lo + w - first;
+      p.u[w] = m[a];
+      p.e[w] = e[a];
+      p.g[w] = g[a];
+      vec = vec && aligned(m[a], 16) && aligned(e[a], 16) && aligned(g[a], 16);
+    }
+    p.table = sk->tables + (size_t)grp * sk->r * sk->c * W;
+    p.d = d;
+    p.nw = nw;
+    p.r = sk->r;
+    p.c = (uint32_t)sk->c;
+    p.cmask = (uint32_t)sk->c - 1;
+    p.rho = rho;
+    p.h = sk->h;
+    cudaError_t err = gs::launch_accumulate_insert(p, W, vec, s);
+    if (err != cudaSuccess) return cuda_fail(err, "accumulate_insert launch");
+  }
+  return GS_OK;
+}
+
+gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float* const* g,
+                    int64_t d, float rho, int64_t k, int64_t* idx, float* vals, float* est,
+                    void* ws, cudaStream_t s) {
+  const size_t bytes = (size_t)sk->groups * sk->r * sk->c * sk->W * sizeof(float) +
+                       (size_t)sk->r * sk->c * sizeof(float);
+  cudaError_t err = cudaMemsetAsync(sk->tables, 0, bytes, s);
+  if (err != cudaSuccess) return cuda_fail(err, "zero tables");
+  GS_TRY(accumulate_insert_impl(sk, 0, sk->workers, m, e, g, d, rho, s));
+  gs::MergeParams mp;
+  mp.tables = sk->tables;
+  mp.merged = sk->merged;
+  mp.cells = (int64_t)sk->r * sk->c;
+  mp.group_stride = (int64_t)sk->r * sk->c * sk->W;
+  mp.P = sk->workers;
+  if ((err = gs::launch_merge(mp, sk->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
+  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, s)) !=
+      cudaSuccess)
+    return cuda_fail(err, "query/top-k launch");
+  gs::GatherParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  for (int p = 0; p < sk->workers; ++p) {
+    gp.u[p] = m[p];
+    gp.e[p] = e[p];
+  }
+  gp.idx = idx;
+  gp.vals = vals;
+  gp.k = k;
+  gp.d = d;
+  gp.P = sk->workers;
+  if ((err = gs::launch_gather_and_zero(gp, s)) != cudaSuccess) return cuda_fail(err, "gather launch");
+  return GS_OK;
+}
+
+gs_status check_worker_arrays(int n, float* const* m, float* const* e, const float* const* g) {
+  if (!m || !e) return fail(GS_ERR_INVALID_ARG, "pointer array is NULL");
+  for (int w = 0; w < n; ++w) {
+    GS_TRY(check_vec(m[w], "momentum[p]"));
+    GS_TRY(check_vec(e[w], "error[p]"));
+    if (g) GS_TRY(check_vec(g[w], "grad[p]"));
+  }
+  return GS_OK;
+}
+
+size_t step_ws_bytes(int64_t d, int64_t k) {
+  return gs::query_topk_workspace_bytes(d, k) + (((size_t)k * 8 + 255) & ~size_t(255)) +
+         (((size_t)k * 4 + 255) & ~size_t(255));
+}
+
+}  // namespace
+
+namespace gs {
+
+DeviceInfo device_info() {
+  static std::mutex mu;
+  static std::unordered_map<int, int> sms_of;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = sms_of.find(dev);
+  if (it == sms_of.end()) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1) sms = 1;
+    it = sms_of.emplace(dev, sms).first;
+  }
+  return DeviceInfo{it->second};
+}
+
+int blocks_per_sm(const void* kernel, int block) {
+  static std::mutex mu;
+  static std::unordered_map<const void*, int> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(kernel);
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, block, 0) != cudaSuccess || n < 1) {
+    cudaGetLastError();
+    n = 1;
+  }
+  cache.emplace(kernel, n);
+  return n;
+}
+
+}  // namespace gs
+
+extern "C" {
+
+gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers, int32_t group_width,
+                           gs_sketch** out) {
+  GS_GUARD_BEGIN
+  if (!out) return fail(GS_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (r < 1 || r > GS_MAX_ROWS) return fail(GS_ERR_INVALID_ARG, "r must lie in [1, 16]");
+  if (c < 1 || c > GS_MAX_COLS) return fail(GS_ERR_INVALID_ARG, "c must lie in [1, 2^26]");
+  if (workers < 1 || workers > GS_MAX_WORKERS) return fail(GS_ERR_INVALID_ARG, "workers must lie in [1, 64]");
+  if (group_width != 0 && group_width != 1 && group_width != 2 && group_width != 4 && group_width != 8)
+    return fail(GS_ERR_INVALID_ARG, "group_width must be 0, 1, 2, 4 or 8");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  const int W = group_width ? group_width : choose_group_width(r, c, workers);
+  const int groups = (workers + W - 1) / W;
+  const size_t table_floats = (size_t)groups * r * c * W;
+  const size_t bytes = (table_floats + (size_t)r * c) * sizeof(float);
+  float* mem = nullptr;
+  e = cudaMalloc(&mem, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(e == cudaErrorMemoryAllocation ? GS_ERR_OOM : GS_ERR_CUDA,
+                std::string("cudaMalloc of ") + std::to_string(bytes) + " bytes: " + cudaGetErrorString(e));
+  }
+  e = cudaMemset(mem, 0, bytes);
+  if (e != cudaSuccess) {
+    cudaFree(mem);
+    return cuda_fail(e, "cudaMemset");
+  }
+  gs_sketch* sk = new gs_sketch;
+  sk->r = r;
+  sk->c = c;
+  sk->workers = workers;
+  sk->W = W;
+  sk->groups = groups;
+  sk->seed = seed;
+  derive_coefficients(r, seed, sk->h);
+  sk->tables = mem;
+  sk->merged = mem + table_floats;
+  sk->device = dev;
+  *out = sk;
+  return ok();
+  GS_GUARD_END
+}
+
+gs_status gs_sketch_destroy(gs_sketch* sk) {
+  if (!sk) return GS_OK;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (prev != sk->device) cudaSetDevice(sk->device);
+  cudaError_t e = cudaFree(sk->tables);
+  if (prev >= 0 && prev != sk->device) cudaSetDevice(prev);
+  delete sk;
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFree");
+  return GS_OK;
+}
+
+gs_status gs_sketch_info(const gs_sketch* sk, int32_t* r, int32_t* c, int32_t* workers, int32_t* group_width) {
+  if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
+  if (r) *r = sk->r;
+  if (c) *c = sk->c;
+  if (workers) *workers = sk->workers;
+  if (group_width) *group_width = sk->W;
+  return GS_OK;
+}
+
+gs_status gs_sketch_coefficients(const gs_sketch* sk, uint64_t* out4r) {
+  if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
+  if (!out4r) return fail(GS_ERR_INVALID_ARG, "out4r is NULL");
+  for (int j = 0; j < sk->r; ++j) {
+    out4r[4 * j + 0] = sk->h.a[j];
+    out4r[4 * j + 1] = sk->h.b[j];
+    out4r[4 * j + 2] = sk->h.a2[j];
+    out4r[4 * j + 3] = sk->h.b2[j];
+  }
+  return GS_OK;
+}
+
+gs_status gs_sketch_zero(gs_sketch* sk, gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  const size_t bytes = ((size_t)sk->groups * sk->r * sk->c * sk->W + (size_t)sk->r * sk->c) * sizeof(float);
+  cudaError_t e = cudaMemsetAsync(sk->tables, 0, bytes, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  return GS_OK;
+}
+
+gs_status gs_accumulate(float* momentum, float* error, const float* grad, int64_t d, float rho, gs_stream stream) {
+  GS_TRY(check_vec(momentum, "momentum"));
+  GS_TRY(check_vec(error, "error"));
+  GS_TRY(check_vec(grad, "grad"));
+  GS_TRY(check_d(d));
+  cudaError_t e = gs::launch_accumulate(momentum, error, grad, d, rho, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "accumulate launch");
+  return GS_OK;
+}
+
+gs_status gs_sketch_insert(gs_sketch* sk, int32_t worker, const float* vec, int64_t d, gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_vec(vec, "vec"));
+  GS_TRY(check_d(d));
+  if (worker < 0 || worker >= sk->workers) return fail(GS_ERR_INVALID_ARG, "worker out of range");
+  gs::InsertParams p;
+  std::memset(&p, 0, sizeof(p));
+  const int W = sk->W;
+  p.e[0] = const_cast<float*>(vec);
+  p.table = sk->tables + (size_t)(worker / W) * sk->r * sk->c * W;
+  p.lane = worker % W;
+  p.d = d;
+  p.nw = 1;
+  p.r = sk->r;
+  p.c = (uint32_t)sk->c;
+  p.cmask = (uint32_t)sk->c - 1;
+  p.h = sk->h;
+  cudaError_t e = gs::launch_insert_lane(p, W, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "insert launch");
+  return GS_OK;
+}
+
+gs_status gs_accumulate_insert(gs_sketch* sk, int32_t first_worker, int32_t n_workers, float* const* momentum,
+                               float* const* error, const float* const* grad, int64_t d, float rho,
+                               gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (n_workers < 1 || first_worker < 0 || first_worker + n_workers > sk->workers)
+    return fail(GS_ERR_INVALID_ARG, "worker range out of bounds");
+  if (first_worker % sk->W != 0) return fail(GS_ERR_INVALID_ARG, "first_worker must be a multiple of the group width");
+  const int end = first_worker + n_workers;
+  if (end % sk->W != 0 && end != sk->workers)
+    return fail(GS_ERR_INVALID_ARG, "the worker range must end on a group boundary or at the last worker");
+  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  GS_TRY(check_worker_arrays(n_workers, momentum, error, grad));
+  return accumulate_insert_impl(sk, first_worker, n_workers, momentum, error, grad, d, rho, as_stream(stream));
+  GS_GUARD_END
+}
+
+gs_status gs_sketch_merge_tree(gs_sketch* sk, int32_t P, gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  if (P < 1 || P > sk->workers) return fail(GS_ERR_INVALID_ARG, "P must lie in [1, workers]");
+  gs::MergeParams mp;
+  mp.tables = sk->tables;
+  mp.merged = sk->merged;
+  mp.cells = (int64_t)sk->r * sk->c;
+  mp.group_stride = (int64_t)sk->r * sk->c * sk->W;
+  mp.P = P;
+  cudaError_t e = gs::launch_merge(mp, sk->W, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+  return GS_OK;
+}
+
+gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = gs::query_topk_workspace_bytes(d, k);
+  return GS_OK;
+}
+
+gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_out, float* est_out,
+                        void* workspace, size_t workspace_bytes, gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  if (est_out) GS_TRY(check_vec(est_out, "est_out"));
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < gs::query_topk_workspace_bytes(d, k))
+    return fail(GS_ERR_INVALID_ARG, "workspace too small: need " + std::to_string(gs::query_topk_workspace_bytes(d, k)));
+  cudaError_t e = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx_out, est_out, workspace,
+                                        as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "query/top-k launch");
+  return GS_OK;
+}
+
+gs_status gs_gather_and_zero(float* const* momentum, float* const* error, int32_t P, int64_t d, const int64_t* idx,
+                             int64_t k, float* vals_out, gs_stream stream) {
+  GS_GUARD_BEGIN
+  if (P < 1 || P > GS_MAX_WORKERS) return fail(GS_ERR_INVALID_ARG, "P must lie in [1, 64]");
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!idx || !aligned(idx, 8)) return fail(GS_ERR_INVALID_ARG, "idx is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals_out, "vals_out"));
+  GS_TRY(check_worker_arrays(P, momentum, error, nullptr));
+  gs::GatherParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  for (int p = 0; p < P; ++p) {
+    gp.u[p] = momentum[p];
+    gp.e[p] = error[p];
+  }
+  gp.idx = idx;
+  gp.vals = vals_out;
+  gp.k = k;
+  gp.d = d;
+  gp.P = P;
+  cudaError_t e = gs::launch_gather_and_zero(gp, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "gather launch");
+  return GS_OK;
+  GS_GUARD_END
+}
+
+gs_status gs_step_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = step_ws_bytes(d, k);
+  return GS_OK;
+}
+
+gs_status gs_step(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad, int64_t d,
+                  float rho, int64_t k, int64_t* idx_out, float* vals_out, float* est_out, void* workspace,
+                  size_t workspace_bytes, gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad));
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals_out, "vals_out"));
+  if (est_out) GS_TRY(check_vec(est_out, "est_out"));
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < gs::query_topk_workspace_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small");
+  return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, est_out, workspace, as_stream(stream));
+  GS_GUARD_END
+}
+
+gs_status gs_step_host(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad_host,
+                       float* const* grad_dev, int64_t d, float rho, int64_t k, int64_t* idx_host, float* vals_host,
+                       void* workspace, size_t workspace_bytes, gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!grad_host || !grad_dev) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  for (int p = 0; p < sk->workers; ++p)
+    if (!grad_host[p]) return fail(GS_ERR_INVALID_ARG, "grad_host[p] is NULL");
+  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad_dev));
+  if (!idx_host || !vals_host) return fail(GS_ERR_INVALID_ARG, "host outputs are NULL");
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < step_ws_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_step_workspace_size");
+  cudaStream_t s = as_stream(stream);
+  const size_t qbytes = gs::query_topk_workspace_bytes(d, k);
+  int64_t* idx_dev = reinterpret_cast<int64_t*>(static_cast<char*>(workspace) + qbytes);
+  float* vals_dev = reinterpret_cast<float*>(reinterpret_cast<char*>(idx_dev) + (((size_t)k * 8 + 255) & ~size_t(255)));
+  for (int p = 0; p < sk->workers; ++p) {
+    cudaError_t e = cudaMemcpyAsync(grad_dev[p], grad_host[p], (size_t)d * sizeof(float), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
+  }
+  GS_TRY(step_impl(sk, momentum, error, grad_dev, d, rho, k, idx_dev, vals_dev, nullptr, workspace, s));
+  cudaError_t e = cudaMemcpyAsync(idx_host, idx_dev, (size_t)k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(vals_host, vals_dev, (size_t)k * sizeof(float), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "result download");
+  return GS_OK;
+  GS_GUARD_END
+}
+
+gs_status gs_hash_eval(const gs_sketch* sk, const int64_t* coords, int64_t n, int32_t* bucket_out, int8_t* sign_out,
+                       gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  if (n < 1) return fail(GS_ERR_INVALID_ARG, "n must be positive");
+  if (!coords || !aligned(coords, 8)) return fail(GS_ERR_INVALID_ARG, "coords is NULL or not 8-byte aligned");
+  if (!bucket_out || !aligned(bucket_out, 4) || !sign_out) return fail(GS_ERR_INVALID_ARG, "output is NULL or misaligned");
+  cudaError_t e = gs::launch_hash_eval(sk->h, sk->r, (uint32_t)sk->c, coords, n, bucket_out, sign_out, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "hash_eval launch");
+  return GS_OK;
+}
+
+gs_status gs_sketch_copy_to_host(const gs_sketch* sk, int32_t worker, float* host_out) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  if (!host_out) return fail(GS_ERR_INVALID_ARG, "host_out is NULL");
+  if (worker < -1 || worker >= sk->workers) return fail(GS_ERR_INVALID_ARG, "worker out of range");
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  const size_t cells = (size_t)sk->r * sk->c;
+  if (worker < 0) {
+    e = cudaMemcpy(host_out, sk->merged, cells * sizeof(float), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+    return GS_OK;
+  }
+  const int W = sk->W;
+  std::vector<float> tmp(cells * W);
+  e = cudaMemcpy(tmp.data(), sk->tables + (size_t)(worker / W) * cells * W, cells * W * sizeof(float),
+                 cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+  const int lane = worker % W;
+  for (size_t q = 0; q < cells; ++q) host_out[q] = tmp[q * W + lane];
+  return GS_OK;
+  GS_GUARD_END
+}
+
+const char* gs_last_error(void) { return g_err.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,126 @@
+// Internal declarations shared by the translation units of the gs-SGD compression library.
+// Device-side Count Sketch hashing over the Mersenne prime 2^61 - 1, kernel parameter
+// blocks and the host-side launcher entry points called by the C ABI in gs_api.cu.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "gs_sketch.h"
+
+namespace gs {
+
+constexpr uint64_t kP61 = (1ull << 61) - 1;
+constexpr int kMaxGroup = 8;        // widest worker group interleaved in one table
+constexpr int kBlock = 256;         // threads per CTA for the streaming kernels
+
+// Hash coefficients of every row: h_j uses (a[j], b[j]); s_j uses (a2[j], b2[j]).
+struct HashCoeffs {
+  uint64_t a[GS_MAX_ROWS], b[GS_MAX_ROWS], a2[GS_MAX_ROWS], b2[GS_MAX_ROWS];
+};
+
+// ---- Mersenne-prime arithmetic ----------------------------------------------------------
+// x mod p is congruent to (x & p) + (x >> 61) because 2^61 = 1 (mod p).
+__device__ __forceinline__ uint64_t fold61(uint64_t x) { return (x & kP61) + (x >> 61); }
+
+// (a*i + b) mod p for a, b < p and i < 2^32.  a is split into 32-bit halves:
+//   a*i = ahi*i*2^32 + alo*i,  and  ahi*i*2^32 = q*2^61 + rem*2^32 = q + rem*2^32 (mod p)
+// with q = (ahi*i) >> 29 and rem = (ahi*i) mod 2^29.  Every partial sum stays below 2^63.
+__device__ __forceinline__ uint64_t affine61(uint64_t a, uint64_t b, uint32_t i) {
+  const uint64_t p0 = (uint64_t)(uint32_t)a * i;          // < 2^64
+  const uint64_t p1 = (uint64_t)(uint32_t)(a >> 32) * i;  // < 2^61
+  uint64_t s = (p1 >> 29) + ((p1 & ((1ull << 29) - 1)) << 32) + fold61(p0) + b;
+  s = fold61(s);                                          // < p + 4
+  return s >= kP61 ? s - kP61 : s;
+}
+
+// x + a mod p for x, a < p: the next coordinate's hash value in the incremental form
+// (a*(i+1) + b) = (a*i + b) + a.
+__device__ __forceinline__ uint64_t step61(uint64_t x, uint64_t a) {
+  x += a;
+  return x >= kP61 ? x - kP61 : x;
+}
+
+template <bool POW2>
+__device__ __forceinline__ uint32_t bucket_of(uint64_t x, uint32_t c, uint32_t cmask) {
+  if (POW2) return (uint32_t)x & cmask;
+  return (uint32_t)(x % (uint64_t)c);
+}
+
+// Sign bit (bit 31 set for s = -1): s_j(i) = -1 when the second hash value is odd.
+__device__ __forceinline__ uint32_t signbit_of(uint64_t y) { return ((uint32_t)y & 1u) << 31; }
+
+__device__ __forceinline__ float apply_sign(float v, uint32_t sbit) {
+  return __uint_as_float(__float_as_uint(v) ^ sbit);
+}
+
+// ---- fp32 reductions into L2-resident tables -------------------------------------------
+__device__ __forceinline__ void red_add_f32(float* p, float v) {
+  asm volatile("red.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+}
+__device__ __forceinline__ void red_add_v2(float* p, float v0, float v1) {
+  asm volatile("red.global.add.v2.f32 [%0], {%1, %2};" ::"l"(p), "f"(v0), "f"(v1) : "memory");
+}
+__device__ __forceinline__ void red_add_v4(float* p, float v0, float v1, float v2, float v3) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(v0), "f"(v1),
+               "f"(v2), "f"(v3)
+               : "memory");
+}
+
+// ---- parameter blocks --------------------------------------------------------------------
+struct InsertParams {
+  float* u[kMaxGroup];
+  float* e[kMaxGroup];
+  const float* g[kMaxGroup];
+  float* table;      // base of the group's interleaved table [r][c][W]
+  int64_t d;
+  int32_t nw;        // lanes of the group carrying a worker in this call
+  int32_t lane;      // single-vector insert: the lane written
+  int32_t r;
+  uint32_t c, cmask;
+  float rho;
+  HashCoeffs h;
+};
+
+struct MergeParams {
+  const float* tables;   // all groups, [group][r][c][W]
+  float* merged;         // [r][c]
+  int64_t cells;         // r*c
+  int64_t group_stride;  // r*c*W floats
+  int32_t P;
+};
+
+struct GatherParams {
+  float* u[GS_MAX_WORKERS];
+  float* e[GS_MAX_WORKERS];
+  const int64_t* idx;
+  float* vals;
+  int64_t k, d;
+  int32_t P;
+};
+
+// ---- launchers (return a cudaError_t from the launch) ------------------------------------
+struct DeviceInfo {
+  int sms;
+};
+DeviceInfo device_info();
+// Resident CTAs per SM for `kernel` at `block` threads (cached per kernel address).
+int blocks_per_sm(const void* kernel, int block);
+
+cudaError_t launch_accumulate(float* u, float* e, const float* g, int64_t d, float rho,
+                              cudaStream_t s);
+cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool vec, cudaStream_t s);
+cudaError_t launch_insert_lane(const InsertParams& p, int W, cudaStream_t s);
+cudaError_t launch_hash_eval(const HashCoeffs& h, int r, uint32_t c, const int64_t* coords,
+                             int64_t n, int32_t* bucket_out, int8_t* sign_out, cudaStream_t s);
+cudaError_t launch_merge(const MergeParams& p, int W, cudaStream_t s);
+cudaError_t launch_gather_and_zero(const GatherParams& p, cudaStream_t s);
+
+size_t query_topk_workspace_bytes(int64_t d, int64_t k);
+cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
+                              int64_t d, int64_t k, int64_t* idx_out, float* est_out,
+                              void* workspace, cudaStream_t s);
+
+inline bool is_pow2(uint32_t c) { return c && !(c & (c - 1)); }
+
+}  // namespace gs

@@ -1,0 +1,259 @@
+// Step 1 (accumulate) and step 2 (Count Sketch insert) of the gs-SGD compression step, and
+// the fused pass that does both while streaming each worker's vectors once.
+//
+// Layout: a group of W simulated workers shares one interleaved table [r][c][W] (fp32), so
+// the W workers' contributions to cell (j, b) are adjacent and one 16-byte vector
+// reduction (red.global.add.v4.f32) updates four of them.  All workers share the hash
+// functions (Sec. III-A: sketches only merge by addition when they do), so the 2r hash
+// values of a coordinate are computed once per group instead of once per worker, and
+// within a thread's four consecutive coordinates in the incremental form x(i+1) = x(i) + a.
+#include "gs_common.cuh"
+
+namespace gs {
+
+namespace {
+
+__device__ __forceinline__ void acc1(float rho, float& u, float& e, float g) {
+  u = __fadd_rn(__fmul_rn(rho, u), g);  // fl(fl(rho*u) + g), never contracted to an FMA
+  e = __fadd_rn(e, u);
+}
+
+__global__ void __launch_bounds__(kBlock) k_accumulate(float* __restrict__ u,
+                                                       float* __restrict__ e,
+                                                       const float* __restrict__ g, int64_t d,
+                                                       float rho, int vec) {
+  const int64_t nq = (d + 3) / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nq; q += stride) {
+    const int64_t i0 = q * 4;
+    if (vec && i0 + 4 <= d) {
+      float4 g4 = __ldcs(reinterpret_cast<const float4*>(g + i0));
+      float4 u4 = __ldcs(reinterpret_cast<const float4*>(u + i0));
+      float4 e4 = __ldcs(reinterpret_cast<const float4*>(e + i0));
+      acc1(rho, u4.x, e4.x, g4.x);
+      acc1(rho, u4.y, e4.y, g4.y);
+      acc1(rho, u4.z, e4.z, g4.z);
+      acc1(rho, u4.w, e4.w, g4.w);
+      __stcs(reinterpret_cast<float4*>(u + i0), u4);
+      __stcs(reinterpret_cast<float4*>(e + i0), e4);
+    } else {
+      for (int t = 0; t < 4 && i0 + t < d; ++t) {
+        float uu = u[i0 + t], ee = e[i0 + t];
+        acc1(rho, uu, ee, g[i0 + t]);
+        u[i0 + t] = uu;
+        e[i0 + t] = ee;
+      }
+    }
+  }
+}
+
+// Load (and with ACC, update and store) four consecutive coordinates of lane w.
+template <bool ACC, bool VEC>
+__device__ __forceinline__ void load_lane(const InsertParams& prm, int w, int64_t i0,
+                                          int64_t d, float (&ev)[4]) {
+  if (VEC && i0 + 4 <= d) {
+    float4 e4 = __ldcs(reinterpret_cast<const float4*>(prm.e[w] + i0));
+    if (ACC) {
+      float4 g4 = __ldcs(reinterpret_cast<const float4*>(prm.g[w] + i0));
+      float4 u4 = __ldcs(reinterpret_cast<const float4*>(prm.u[w] + i0));
+      acc1(prm.rho, u4.x, e4.x, g4.x);
+      acc1(prm.rho, u4.y, e4.y, g4.y);
+      acc1(prm.rho, u4.z, e4.z, g4.z);
+      acc1(prm.rho, u4.w, e4.w, g4.w);
+      __stcs(reinterpret_cast<float4*>(prm.u[w] + i0), u4);
+      __stcs(reinterpret_cast<float4*>(prm.e[w] + i0), e4);
+    }
+    ev[0] = e4.x;
+    ev[1] = e4.y;
+    ev[2] = e4.z;
+    ev[3] = e4.w;
+  } else {
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      ev[t] = 0.f;
+      if (i0 + t < d) {
+        float ee = prm.e[w][i0 + t];
+        if (ACC) {
+          float uu = prm.u[w][i0 + t];
+          acc1(prm.rho, uu, ee, prm.g[w][i0 + t]);
+          prm.u[w][i0 + t] = uu;
+          prm.e[w][i0 + t] = ee;
+        }
+        ev[t] = ee;
+      }
+    }
+  }
+}
+
+// One thread = four consecutive coordinates of every worker in the group.
+//   ACC: accumulate (u, e update) before inserting e; otherwise insert e as given.
+//   VEC: all vectors 16-byte aligned (float4 path for full quads).
+//   POW2: c is a power of two (bucket = x & (c - 1)).
+template <int W, bool ACC, bool VEC, bool POW2>
+__global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_constant__ InsertParams prm) {
+  const int64_t d = prm.d;
+  const int64_t nq = (d + 3) / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nq; q += stride) {
+    const int64_t i0 = q * 4;
+    float ev[W][4];
+#pragma unroll
+    for (int w = 0; w < W; ++w) {
+      if (w < prm.nw) {
+        load_lane<ACC, VEC>(prm, w, i0, d, ev[w]);
+      } else {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) ev[w][t] = 0.f;
+      }
+    }
+    const int tmax = (d - i0 < 4) ? (int)(d - i0) : 4;
+#pragma unroll 1
+    for (int j = 0; j < prm.r; ++j) {
+      const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
+      uint64_t x = affine61(a, prm.h.b[j], (uint32_t)i0);
+      uint64_t y = affine61(a2, prm.h.b2[j], (uint32_t)i0);
+      float* row = prm.table + (size_t)j * prm.c * W;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        if (t < tmax) {
+          const uint32_t bk = bucket_of<POW2>(x, prm.c, prm.cmask);
+          const uint32_t sb = signbit_of(y);
+          float* cell = row + (size_t)bk * W;
+          if (W == 1) {
+            red_add_f32(cell, apply_sign(ev[0][t], sb));
+          } else if (W == 2) {
+            red_add_v2(cell, apply_sign(ev[0][t], sb), apply_sign(ev[W > 1 ? 1 : 0][t], sb));
+          } else {
+#pragma unroll
+            for (int w4 = 0; w4 < W; w4 += 4) {
+              red_add_v4(cell + w4, apply_sign(ev[w4][t], sb),
+                         apply_sign(ev[w4 + 1 < W ? w4 + 1 : 0][t], sb),
+                         apply_sign(ev[w4 + 2 < W ? w4 + 2 : 0][t], sb),
+                         apply_sign(ev[w4 + 3 < W ? w4 + 3 : 0][t], sb));
+            }
+          }
+          if (t < 3) {
+            x = step61(x, a);
+            y = step61(y, a2);
+          }
+        }
+      }
+    }
+  }
+}
+
+// Insert one vector (prm.e[0]) into lane prm.lane of a W-wide group table.
+template <bool POW2>
+__global__ void __launch_bounds__(kBlock) k_insert_lane(const __grid_constant__ InsertParams prm, int W) {
+  const int64_t d = prm.d;
+  const int64_t nq = (d + 3) / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const float* v = prm.e[0];
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nq; q += stride) {
+    const int64_t i0 = q * 4;
+    const int tmax = (d - i0 < 4) ? (int)(d - i0) : 4;
+    float ev[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) ev[t] = (t < tmax) ? v[i0 + t] : 0.f;
+#pragma unroll 1
+    for (int j = 0; j < prm.r; ++j) {
+      const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
+      uint64_t x = affine61(a, prm.h.b[j], (uint32_t)i0);
+      uint64_t y = affine61(a2, prm.h.b2[j], (uint32_t)i0);
+      float* row = prm.table + (size_t)j * prm.c * W + prm.lane;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        if (t < tmax) {
+          const uint32_t bk = bucket_of<POW2>(x, prm.c, prm.cmask);
+          red_add_f32(row + (size_t)bk * W, apply_sign(ev[t], signbit_of(y)));
+          x = step61(x, a);
+          y = step61(y, a2);
+        }
+      }
+    }
+  }
+}
+
+__global__ void k_hash_eval(const __grid_constant__ HashCoeffs h, int r, uint32_t c,
+                            const int64_t* __restrict__ coords, int64_t n,
+                            int32_t* __restrict__ bucket_out, int8_t* __restrict__ sign_out) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += stride) {
+    const int64_t i = coords[t];
+    const bool ok = (i >= 0 && i < (1ll << 31));
+    for (int j = 0; j < r; ++j) {
+      if (ok) {
+        const uint64_t x = affine61(h.a[j], h.b[j], (uint32_t)i);
+        const uint64_t y = affine61(h.a2[j], h.b2[j], (uint32_t)i);
+        bucket_out[(int64_t)j * n + t] = (int32_t)(x % (uint64_t)c);
+        sign_out[(int64_t)j * n + t] = (y & 1u) ? (int8_t)-1 : (int8_t)1;
+      } else {
+        bucket_out[(int64_t)j * n + t] = -1;
+        sign_out[(int64_t)j * n + t] = 0;
+      }
+    }
+  }
+}
+
+template <typename K>
+int grid_for(K kernel, int64_t work_items, int block) {
+  const int64_t need = (work_items + block - 1) / block;
+  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)kernel, block);
+  return (int)(need < 1 ? 1 : (need < cap ? need : cap));
+}
+
+template <int W, bool ACC, bool VEC, bool POW2>
+cudaError_t launch_ai_t(const InsertParams& p, cudaStream_t s) {
+  auto kern = k_accumulate_insert<W, ACC, VEC, POW2>;
+  const int grid = grid_for(kern, (p.d + 3) / 4, kBlock);
+  kern<<<grid, kBlock, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <int W, bool ACC>
+cudaError_t launch_ai_w(const InsertParams& p, bool vec, cudaStream_t s) {
+  const bool pow2 = is_pow2(p.c);
+  if (vec) return pow2 ? launch_ai_t<W, ACC, true, true>(p, s) : launch_ai_t<W, ACC, true, false>(p, s);
+  return pow2 ? launch_ai_t<W, ACC, false, true>(p, s) : launch_ai_t<W, ACC, false, false>(p, s);
+}
+
+}  // namespace
+
+cudaError_t launch_accumulate(float* u, float* e, const float* g, int64_t d, float rho,
+                              cudaStream_t s) {
+  const bool vec = ((reinterpret_cast<uintptr_t>(u) | reinterpret_cast<uintptr_t>(e) |
+                     reinterpret_cast<uintptr_t>(g)) & 15u) == 0;
+  const int grid = grid_for(k_accumulate, (d + 3) / 4, kBlock);
+  k_accumulate<<<grid, kBlock, 0, s>>>(u, e, g, d, rho, vec ? 1 : 0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool vec, cudaStream_t s) {
+  switch (W) {
+    case 1: return launch_ai_w<1, true>(p, vec, s);
+    case 2: return launch_ai_w<2, true>(p, vec, s);
+    case 4: return launch_ai_w<4, true>(p, vec, s);
+    case 8: return launch_ai_w<8, true>(p, vec, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_insert_lane(const InsertParams& p, int W, cudaStream_t s) {
+  if (is_pow2(p.c)) {
+    const int grid = grid_for(k_insert_lane<true>, (p.d + 3) / 4, kBlock);
+    k_insert_lane<true><<<grid, kBlock, 0, s>>>(p, W);
+  } else {
+    const int grid = grid_for(k_insert_lane<false>, (p.d + 3) / 4, kBlock);
+    k_insert_lane<false><<<grid, kBlock, 0, s>>>(p, W);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_hash_eval(const HashCoeffs& h, int r, uint32_t c, const int64_t* coords,
+                             int64_t n, int32_t* bucket_out, int8_t* sign_out, cudaStream_t s) {
+  const int grid = grid_for(k_hash_eval, n, kBlock);
+  k_hash_eval<<<grid, kBlock, 0, s>>>(h, r, c, coords, n, bucket_out, sign_out);
+  return cudaGetLastError();
+}
+
+}  // namespace gs

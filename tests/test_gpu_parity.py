@@ -1,0 +1,274 @@
+"""GPU parity: every call of the C ABI against the CPU oracle (run on a GB300).
+
+Sizes span several CUDA tiles and ragged tails; the workload shapes are those of the
+tiny (d = 2^20, P = 4) and ResNet-18-sized (d = 11,173,962, P = 8) configurations, plus
+edge cases (d = 1, k = 1, k = d, c = 1, odd and even r, P not a power of two, every group
+width, misaligned vectors).
+"""
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle  # noqa: E402
+import workloads  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+P61 = (1 << 61) - 1
+
+
+@pytest.fixture(scope="module")
+def gs():
+    import paper_2108_06004_gb300 as lib
+    lib.load_library()
+    torch.cuda.set_device(0)
+    return lib
+
+
+@pytest.fixture(scope="module")
+def H(gs):
+    from tests import gpu_harness
+    return gpu_harness
+
+
+def _dev(x):
+    return torch.from_numpy(np.ascontiguousarray(x)).cuda()
+
+
+# ---- hash family ------------------------------------------------------------------------
+
+@pytest.mark.parametrize("r,c,seed", [(5, 1 << 14, 20210813), (7, 1 << 20, 3), (3, 1000, 99), (16, 1, 0),
+                                      (1, (1 << 26), 2**64 - 1)])
+def test_coefficients_and_hashes_bit_exact(gs, r, c, seed):
+    sk = gs.gs_sketch_create(r, c, seed, 1)
+    try:
+        coeffs = gs.gs_sketch_coefficients(sk)
+        assert tuple(coeffs) == tuple(oracle.derive_coefficients(r, seed))
+        rng = np.random.default_rng(seed % 1000)
+        coords = np.concatenate([np.arange(1 << 16), [2**31 - 1, 2**31 - 2, 2**30, 11173961],
+                                 rng.integers(0, 2**31, 200_000)]).astype(np.int64)
+        n = coords.size
+        bk = torch.empty(r * n, dtype=torch.int32, device="cuda")
+        sg = torch.empty(r * n, dtype=torch.int8, device="cuda")
+        gs.gs_hash_eval(sk, _dev(coords), n, bk, sg)
+        want_b, want_s = oracle.hash_rows(coeffs, c, coords.astype(np.uint64))
+        assert np.array_equal(bk.cpu().numpy().reshape(r, n), want_b)
+        assert np.array_equal(sg.cpu().numpy().reshape(r, n), want_s)
+        for t in (0, 1, n - 1, n - 2):
+            for j in range(r):
+                assert want_b[j, t] == oracle.bucket_exact(coeffs[0][j], coeffs[1][j], c, int(coords[t]))
+        bad = _dev(np.array([-1, 2**31], dtype=np.int64))
+        bk2 = torch.empty(r * 2, dtype=torch.int32, device="cuda")
+        sg2 = torch.empty(r * 2, dtype=torch.int8, device="cuda")
+        gs.gs_hash_eval(sk, bad, 2, bk2, sg2)
+        assert np.all(bk2.cpu().numpy() == -1) and np.all(sg2.cpu().numpy() == 0)
+    finally:
+        gs.gs_sketch_destroy(sk)
+
+
+# ---- step 1 ------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("d,offset", [(1, 0), (7, 0), (1_000_003, 0), (1_000_003, 1), (4096 * 152 * 3 + 2, 3)])
+def test_accumulate_bit_exact(gs, d, offset):
+    rng = np.random.default_rng(d + offset)
+    mk = lambda: (rng.standard_normal(d) * 10.0 ** rng.integers(-30, 6, d)).astype(np.float32)
+    u, e, g = mk(), mk(), mk()
+    bufs = [torch.zeros(d + 4, dtype=torch.float32, device="cuda") for _ in range(3)]
+    views = [b[offset:offset + d] for b in bufs]
+    for v, x in zip(views, (u, e, g)):
+        v.copy_(torch.from_numpy(x))
+    for rho in (0.9, 0.0, 0.5):
+        gs.gs_accumulate(views[0], views[1], views[2], d, rho)
+        u, e = oracle.accumulate(u, e, g, rho)
+        assert np.array_equal(views[0].cpu().numpy().view(np.uint32), u.view(np.uint32))
+        assert np.array_equal(views[1].cpu().numpy().view(np.uint32), e.view(np.uint32))
+    for b in bufs:  # guard cells outside the view untouched
+        assert torch.all(b[:offset] == 0) and torch.all(b[offset + d:] == 0)
+
+
+# ---- step 2 ------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("W,worker,P", [(1, 0, 1), (2, 1, 2), (4, 2, 3), (8, 5, 8), (8, 7, 13)])
+def test_single_vector_insert(gs, H, W, worker, P):
+    d, r, c, seed = 300_001, 5, 1 << 12, 5
+    rng = np.random.default_rng(W)
+    x = (rng.standard_normal(d) * 1e-3).astype(np.float32)
+    sk = gs.gs_sketch_create(r, c, seed, P, W)
+    try:
+        gs.gs_sketch_insert(sk, worker, _dev(x), d)
+        run = H.GpuRun(sk, [], [], d, 1, 0.9, None, None, None, None)
+        tabs = H.worker_tables(run, P, r, c)
+        T, A = oracle.sketch(x, oracle.derive_coefficients(r, seed), c)
+        H.check_cells(tabs[worker], T, A, "inserted table")
+        for p in range(P):
+            if p != worker:
+                assert np.all(tabs[p] == 0)
+    finally:
+        gs.gs_sketch_destroy(sk)
+
+
+@pytest.mark.parametrize("P,W,d,r,c", [(1, 1, 70_001, 3, 1 << 10), (3, 4, 123_457, 5, 1000),
+                                       (5, 8, 200_003, 4, 1 << 13), (8, 2, 65_536, 5, 1 << 12),
+                                       (8, 8, 400_000, 7, 1 << 14), (16, 8, 50_001, 5, 777)])
+def test_accumulate_insert_merge(gs, H, P, W, d, r, c):
+    seed = P * 1000 + W
+    rng = np.random.default_rng(seed)
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, 1, seed, rho=0.9, group_width=W)
+    try:
+        assert gs.gs_sketch_info(run.sketch)["group_width"] == W
+        us = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        es = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        gr = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        for p in range(P):
+            run.us[p].copy_(torch.from_numpy(us[p]))
+            run.es[p].copy_(torch.from_numpy(es[p]))
+        gdev = [_dev(g) for g in gr]
+        # two calls covering the workers in group-aligned pieces
+        split = min(P, W) if P > W else P
+        gs.gs_accumulate_insert(run.sketch, 0, run.us[:split], run.es[:split], gdev[:split], d, 0.9)
+        if split < P:
+            gs.gs_accumulate_insert(run.sketch, split, run.us[split:], run.es[split:], gdev[split:], d, 0.9)
+        gs.gs_sketch_merge_tree(run.sketch, P)
+        tabs = H.worker_tables(run, P, r, c)
+        merged = H.merged_table(run, r, c)
+        Ts, As = [], []
+        for p in range(P):
+            u1, e1 = oracle.accumulate(us[p], es[p], gr[p], 0.9)
+            assert np.array_equal(H.host(run.us[p]).view(np.uint32), u1.view(np.uint32))
+            assert np.array_equal(H.host(run.es[p]).view(np.uint32), e1.view(np.uint32))
+            T, A = oracle.sketch(e1, coeffs, c)
+            H.check_cells(tabs[p], T, A, f"worker {p}")
+            Ts.append(T)
+            As.append(A)
+        assert np.array_equal(merged, H.fp32_tree(tabs)), "merge is not the fp32 tree of the worker tables"
+        H.check_cells(merged, oracle.merge_tree(Ts), oracle.merge_tree(As), "merged")
+        for Pm in range(1, P + 1):  # partial merges follow the same schedule
+            gs.gs_sketch_merge_tree(run.sketch, Pm)
+            assert np.array_equal(H.merged_table(run, r, c), H.fp32_tree(tabs[:Pm]))
+    finally:
+        run.close()
+
+
+# ---- steps 4-5 ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("d,r,c,k", [(1, 5, 64, 1), (10, 3, 1, 4), (1000, 1, 1, 1000), (100_003, 5, 4096, 1),
+                                     (100_003, 4, 4096, 333), (1 << 20, 5, 1 << 14, 1000),
+                                     (500_000, 7, 3000, 500_000), (2_000_001, 15, 1 << 16, 2000)])
+def test_query_topk(gs, H, d, r, c, k):
+    seed = d + r + c + k
+    rng = np.random.default_rng(seed % 2**32)
+    coeffs = oracle.derive_coefficients(r, seed)
+    x = (rng.standard_normal(d) * 1e-3).astype(np.float32)
+    x[rng.choice(d, max(1, d // 500), replace=False)] *= 100
+    run = H.new_run(1, d, r, c, k, seed)
+    try:
+        gs.gs_sketch_insert(run.sketch, 0, _dev(x), d)
+        gs.gs_sketch_merge_tree(run.sketch, 1)
+        ws = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        gs.gs_query_topk(run.sketch, d, k, run.idx, run.est, ws)
+        est, idx = H.host(run.est), H.host(run.idx)
+        T, A = oracle.sketch(x, coeffs, c)
+        est_o = oracle.query(T, coeffs, d)
+        band = oracle.cell_band(A, coeffs, np.arange(d))
+        assert np.all(np.abs(est.astype(np.float64) - est_o) <= band)
+        H.check_selection_exact(idx, est, k)
+        H.check_topk_set(idx, oracle.topk(est_o, k), est_o, band, k, d)
+        # without est_out the same indices come out
+        idx2 = torch.empty(k, dtype=torch.int64, device="cuda")
+        gs.gs_query_topk(run.sketch, d, k, idx2, None, ws)
+        assert np.array_equal(H.host(idx2), idx)
+    finally:
+        run.close()
+
+
+def test_topk_all_ties_and_zeros(gs, H):
+    d, r, c, k = 50_000, 5, 256, 1234
+    run = H.new_run(1, d, r, c, k, 1)
+    try:
+        ws = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        gs.gs_sketch_merge_tree(run.sketch, 1)           # all-zero sketch: est = 0 everywhere
+        gs.gs_query_topk(run.sketch, d, k, run.idx, run.est, ws)
+        assert np.array_equal(H.host(run.idx), np.arange(k))
+    finally:
+        run.close()
+
+
+# ---- step 6 ------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("P,d,k", [(1, 10, 10), (4, 1_000_003, 1000), (64, 20_000, 777)])
+def test_gather_and_zero(gs, P, d, k):
+    rng = np.random.default_rng(P)
+    us = [(rng.standard_normal(d)).astype(np.float32) for _ in range(P)]
+    es = [(rng.standard_normal(d)).astype(np.float32) for _ in range(P)]
+    idx = np.sort(rng.choice(d, k, replace=False)).astype(np.int64)
+    ud, ed = [_dev(u) for u in us], [_dev(e) for e in es]
+    vals = torch.empty(k, dtype=torch.float32, device="cuda")
+    gs.gs_gather_and_zero(ud, ed, d, _dev(idx), k, vals)
+    v, us2, es2 = oracle.gather_and_zero(us, es, idx)
+    stack = np.stack([e[idx].astype(np.float64) for e in es])
+    assert np.all(np.abs(vals.cpu().numpy() - v) <= (P - 1) * 2.0**-24 * np.abs(stack).sum(0) * 1.000001)
+    # the fp32 sum in worker order, exactly
+    ref = np.zeros(k, np.float32)
+    for e in es:
+        ref = (ref + e[idx]).astype(np.float32)
+    assert np.array_equal(vals.cpu().numpy(), ref)
+    for p in range(P):
+        assert np.array_equal(ud[p].cpu().numpy(), us2[p]) and np.array_equal(ed[p].cpu().numpy(), es2[p])
+
+
+def test_gather_skips_out_of_range(gs):
+    d = 100
+    u = [torch.ones(d, device="cuda")]
+    e = [torch.ones(d, device="cuda")]
+    idx = _dev(np.array([-5, 3, 100, 2**40], dtype=np.int64))
+    vals = torch.empty(4, device="cuda")
+    gs.gs_gather_and_zero(u, e, d, idx, 4, vals)
+    v = vals.cpu().numpy()
+    assert np.isnan(v[0]) and v[1] == 1.0 and np.isnan(v[2]) and np.isnan(v[3])
+    assert float(u[0].sum()) == d - 1 and float(e[0][3]) == 0.0
+
+
+# ---- whole steps -------------------------------------------------------------------------
+
+def _run_steps(gs, H, w, d, steps, c=None, k=None, r=None, P=None, group_width=0, seed=2021):
+    P = P or w.P
+    r = r or w.r
+    c = c or w.c
+    k = k or w.k
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho, group_width=group_width)
+    nsym = 0
+    try:
+        for t in range(steps):
+            grads = workloads.make_gradients(w, t, range(P), d=d)
+            gdev = [_dev(g) for g in grads]
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            H.gpu_step(run, gdev)
+            torch.cuda.synchronize()
+            res = oracle.step(us0, es0, grads, w.rho, coeffs, c, k)
+            nsym += H.compare_step(res, coeffs, [H.host(u) for u in run.us], [H.host(e) for e in run.es],
+                                   H.host(run.idx), H.host(run.vals), H.host(run.est), k,
+                                   H.worker_tables(run, P, r, c), H.merged_table(run, r, c))
+    finally:
+        run.close()
+    return nsym
+
+
+def test_steps_tiny_config(gs, H):
+    w = workloads.get_config("tiny-2^20")
+    _run_steps(gs, H, w, w.d, w.steps)
+
+
+@pytest.mark.parametrize("P,r,c,k,W", [(5, 4, 1000, 777, 0), (6, 3, 4099, 50, 2), (3, 5, 1 << 12, 1, 1)])
+def test_steps_ragged(gs, H, P, r, c, k, W):
+    w = workloads.get_config("resnet18")
+    _run_steps(gs, H, w, 100_003, 2, c=c, k=k, r=r, P=P, group_width=W)
+
+
+def test_steps_resnet18_full_size(gs, H):
+    w = workloads.get_config("resnet18")
+    _run_steps(gs, H, w, w.d, 2)
