@@ -64,9 +64,11 @@ typedef void* gs_stream;            /* a cudaStream_t */
  * drawn from `seed` (Sec. III-A: sketches combine by addition only when they share their
  * hash functions), plus the merged r x c table that gs_sketch_merge_tree writes.
  * All tables start at zero.  Worker tables are stored interleaved in groups of
- * `group_width` workers ([group][r][c][group_width] fp32) so that one 16-byte vector
- * reduction updates four workers' cells at once; group_width 0 lets the library choose
- * (the widest of 8, 4, 2, 1 whose group table fits a fixed L2-sized budget).
+ * `group_width` workers ([group][r][c][group_width] fp32) so that the group's values of a
+ * cell are adjacent and are updated by 16-byte vector reductions; group_width 0 lets the
+ * library choose (up to 8, no wider than the worker count rounded up to a power of two,
+ * halved while one table row exceeds a 64 MiB L2 budget).  The fused insert updates as many
+ * rows per pass as fit that budget.
  * On success *out owns device memory released by gs_sketch_destroy.
  * Errors: GS_ERR_INVALID_ARG (sizes, group_width not in {0,1,2,4,8}, out NULL),
  *         GS_ERR_OOM (allocation failed), GS_ERR_CUDA.  Synchronous. */
@@ -76,9 +78,10 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
 /* Release a sketch and its device memory.  NULL is accepted.  Synchronous. */
 gs_status gs_sketch_destroy(gs_sketch* sketch);
 
-/* Shape query: any output pointer may be NULL. */
+/* Shape query: any output pointer may be NULL.  rows_per_pass is the number of rows the
+ * fused insert updates per pass over the vectors. */
 gs_status gs_sketch_info(const gs_sketch* sketch, int32_t* r, int32_t* c, int32_t* workers,
-                         int32_t* group_width);
+                         int32_t* group_width, int32_t* rows_per_pass);
 
 /* Host copy of the hash coefficients: out4r[4*j + {0,1,2,3}] = a_j, b_j, a'_j, b'_j
  * (host array of 4*r uint64).  Synchronous, no device work. */
@@ -110,7 +113,9 @@ gs_status gs_sketch_insert(gs_sketch* sketch, int32_t worker, const float* vec, 
  * pointer arrays are HOST arrays of n_workers DEVICE pointers.  first_worker must be a
  * multiple of the group width, and the range must end on a group boundary or at the
  * last worker.  Per worker the result equals gs_accumulate followed by gs_sketch_insert
- * (up to the order of the fp32 atomic additions in the cells). */
+ * (up to the order of the fp32 atomic additions in the cells).  When the table is inserted
+ * in several row passes, the first pass also accumulates and the later ones re-read the
+ * updated error vectors. */
 gs_status gs_accumulate_insert(gs_sketch* sketch, int32_t first_worker, int32_t n_workers,
                                float* const* momentum, float* const* error,
                                const float* const* grad, int64_t d, float rho,

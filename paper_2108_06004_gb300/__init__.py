@@ -36,7 +36,7 @@ SIGNATURES = {
     "gs_sketch_create": [_i32, _i32, _u64, _i32, _i32, ctypes.POINTER(_vp)],
     "gs_sketch_destroy": [_vp],
     "gs_sketch_info": [_vp, ctypes.POINTER(_i32), ctypes.POINTER(_i32), ctypes.POINTER(_i32),
-                       ctypes.POINTER(_i32)],
+                       ctypes.POINTER(_i32), ctypes.POINTER(_i32)],
     "gs_sketch_coefficients": [_vp, ctypes.POINTER(_u64)],
     "gs_sketch_zero": [_vp, _vp],
     "gs_accumulate": [_vp, _vp, _vp, _i64, _f32, _vp],
@@ -118,10 +118,11 @@ def gs_sketch_destroy(sketch: int) -> None:
 
 
 def gs_sketch_info(sketch: int) -> dict:
-    r, c, w, g = _i32(), _i32(), _i32(), _i32()
+    r, c, w, g, rp = _i32(), _i32(), _i32(), _i32(), _i32()
     _check(load_library().gs_sketch_info(sketch, ctypes.byref(r), ctypes.byref(c), ctypes.byref(w),
-                                         ctypes.byref(g)), "gs_sketch_info")
-    return {"r": r.value, "c": c.value, "workers": w.value, "group_width": g.value}
+                                         ctypes.byref(g), ctypes.byref(rp)), "gs_sketch_info")
+    return {"r": r.value, "c": c.value, "workers": w.value, "group_width": g.value,
+            "rows_per_pass": rp.value}
 
 
 def gs_sketch_coefficients(sketch: int):

@@ -11,6 +11,7 @@
 
 struct gs_sketch {
   int32_t r, c, workers, W, groups;
+  int32_t rows_per_pass;  // rows inserted per pass of the fused kernel (table slice <= L2 budget)
   uint64_t seed;
   gs::HashCoeffs h;
   float* tables;  // groups * r*c*W
@@ -57,15 +58,25 @@ void derive_coefficients(int r, uint64_t seed, gs::HashCoeffs& h) {
   }
 }
 
-constexpr size_t kGroupBudgetBytes = size_t(64) << 20;  // interleaved group table kept L2-sized
+// The slice of a group table that one insert pass updates is kept within this many bytes, so
+// that the table stays resident in the 126 MB L2 while g, u and e stream past it.
+constexpr size_t kL2BudgetBytes = size_t(64) << 20;
 
-int choose_group_width(int r, int c, int workers) {
-  int cap = 1;
-  while (cap < workers && cap < gs::kMaxGroup) cap *= 2;
-  for (int W = cap; W > 1; W /= 2) {
-    if ((size_t)r * (size_t)c * (size_t)W * sizeof(float) <= kGroupBudgetBytes) return W;
-  }
-  return 1;
+// Widest group (up to 8, not wider than the worker count rounded up to a power of two) whose
+// single table row fits the budget.
+int choose_group_width(int c, int workers) {
+  int W = 1;
+  while (W < workers && W < gs::kMaxGroup) W *= 2;
+  while (W > 1 && (size_t)c * (size_t)W * sizeof(float) > kL2BudgetBytes) W /= 2;
+  return W;
+}
+
+int choose_rows_per_pass(int r, int c, int W) {
+  const size_t row_bytes = (size_t)c * (size_t)W * sizeof(float);
+  size_t n = kL2BudgetBytes / row_bytes;
+  if (n < 1) n = 1;
+  if (n > (size_t)r) n = (size_t)r;
+  return (int)n;
 }
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
@@ -136,8 +147,14 @@ gs_status accumulate_insert_impl(gs_sketch* sk, int32_t first, int32_t n, float*
     p.cmask = (uint32_t)sk->c - 1;
     p.rho = rho;
     p.h = sk->h;
-    cudaError_t err = gs::launch_accumulate_insert(p, W, vec, s);
-    if (err != cudaSuccess) return cuda_fail(err, "accumulate_insert launch");
+    // first pass: accumulate and insert rows [0, rows_per_pass); later passes insert the
+    // remaining rows from the updated error vectors
+    for (int j0 = 0; j0 < sk->r; j0 += sk->rows_per_pass) {
+      p.j0 = j0;
+      p.j1 = (j0 + sk->rows_per_pass < sk->r) ? j0 + sk->rows_per_pass : sk->r;
+      cudaError_t err = gs::launch_accumulate_insert(p, W, j0 == 0, vec, s);
+      if (err != cudaSuccess) return cuda_fail(err, "accumulate_insert launch");
+    }
   }
   return GS_OK;
 }
@@ -241,7 +258,7 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-  const int W = group_width ? group_width : choose_group_width(r, c, workers);
+  const int W = group_width ? group_width : choose_group_width(c, workers);
   const int groups = (workers + W - 1) / W;
   const size_t table_floats = (size_t)groups * r * c * W;
   const size_t bytes = (table_floats + (size_t)r * c) * sizeof(float);
@@ -263,6 +280,7 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   sk->workers = workers;
   sk->W = W;
   sk->groups = groups;
+  sk->rows_per_pass = choose_rows_per_pass(r, c, W);
   sk->seed = seed;
   derive_coefficients(r, seed, sk->h);
   sk->tables = mem;
@@ -285,12 +303,14 @@ gs_status gs_sketch_destroy(gs_sketch* sk) {
   return GS_OK;
 }
 
-gs_status gs_sketch_info(const gs_sketch* sk, int32_t* r, int32_t* c, int32_t* workers, int32_t* group_width) {
+gs_status gs_sketch_info(const gs_sketch* sk, int32_t* r, int32_t* c, int32_t* workers, int32_t* group_width,
+                         int32_t* rows_per_pass) {
   if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
   if (r) *r = sk->r;
   if (c) *c = sk->c;
   if (workers) *workers = sk->workers;
   if (group_width) *group_width = sk->W;
+  if (rows_per_pass) *rows_per_pass = sk->rows_per_pass;
   return GS_OK;
 }
 
@@ -338,6 +358,8 @@ gs_status gs_sketch_insert(gs_sketch* sk, int32_t worker, const float* vec, int6
   p.d = d;
   p.nw = 1;
   p.r = sk->r;
+  p.j0 = 0;
+  p.j1 = sk->r;
   p.c = (uint32_t)sk->c;
   p.cmask = (uint32_t)sk->c - 1;
   p.h = sk->h;

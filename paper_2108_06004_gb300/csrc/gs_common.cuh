@@ -77,6 +77,7 @@ struct InsertParams {
   int32_t nw;        // lanes of the group carrying a worker in this call
   int32_t lane;      // single-vector insert: the lane written
   int32_t r;
+  int32_t j0, j1;    // rows inserted by this launch: [j0, j1)
   uint32_t c, cmask;
   float rho;
   HashCoeffs h;
@@ -109,7 +110,8 @@ int blocks_per_sm(const void* kernel, int block);
 
 cudaError_t launch_accumulate(float* u, float* e, const float* g, int64_t d, float rho,
                               cudaStream_t s);
-cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool vec, cudaStream_t s);
+// acc: accumulate (read g, u, e; write u, e) before inserting; otherwise insert e as it is.
+cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool acc, bool vec, cudaStream_t s);
 cudaError_t launch_insert_lane(const InsertParams& p, int W, cudaStream_t s);
 cudaError_t launch_hash_eval(const HashCoeffs& h, int r, uint32_t c, const int64_t* coords,
                              int64_t n, int32_t* bucket_out, int8_t* sign_out, cudaStream_t s);

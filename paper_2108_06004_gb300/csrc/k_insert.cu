@@ -2,11 +2,18 @@
 // the fused pass that does both while streaming each worker's vectors once.
 //
 // Layout: a group of W simulated workers shares one interleaved table [r][c][W] (fp32), so
-// the W workers' contributions to cell (j, b) are adjacent and one 16-byte vector
-// reduction (red.global.add.v4.f32) updates four of them.  All workers share the hash
+// the W workers' contributions to cell (j, b) are adjacent.  All workers share the hash
 // functions (Sec. III-A: sketches only merge by addition when they do), so the 2r hash
-// values of a coordinate are computed once per group instead of once per worker, and
-// within a thread's four consecutive coordinates in the incremental form x(i+1) = x(i) + a.
+// values of a coordinate serve every worker of the group; a thread evaluates them for
+// four consecutive coordinates, the later three in the incremental form x(i+1) = x(i) + a.
+//
+// L2 reductions are the bound of this pass (random reductions run at a fixed rate of
+// requests, whatever their width up to 16 bytes, and the load-store unit merges the
+// requests of one warp instruction that fall in the same sector).  So for W >= 4 a group of
+// G = W/4 adjacent lanes shares one coordinate quad, each lane owns four workers, and one
+// warp instruction writes whole W*4-byte cells with 16-byte vector reductions
+// (red.global.add.v4.f32).  For tables larger than the L2 budget the rows are inserted in
+// passes over row ranges: the first pass accumulates, later passes only re-read e.
 #include "gs_common.cuh"
 
 namespace gs {
@@ -85,7 +92,7 @@ __device__ __forceinline__ void load_lane(const InsertParams& prm, int w, int64_
   }
 }
 
-// One thread = four consecutive coordinates of every worker in the group.
+// W <= 2: one thread = four consecutive coordinates of every worker in the group.
 //   ACC: accumulate (u, e update) before inserting e; otherwise insert e as given.
 //   VEC: all vectors 16-byte aligned (float4 path for full quads).
 //   POW2: c is a power of two (bucket = x & (c - 1)).
@@ -108,7 +115,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_const
     }
     const int tmax = (d - i0 < 4) ? (int)(d - i0) : 4;
 #pragma unroll 1
-    for (int j = 0; j < prm.r; ++j) {
+    for (int j = prm.j0; j < prm.j1; ++j) {
       const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
       uint64_t x = affine61(a, prm.h.b[j], (uint32_t)i0);
       uint64_t y = affine61(a2, prm.h.b2[j], (uint32_t)i0);
@@ -121,21 +128,58 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_const
           float* cell = row + (size_t)bk * W;
           if (W == 1) {
             red_add_f32(cell, apply_sign(ev[0][t], sb));
-          } else if (W == 2) {
-            red_add_v2(cell, apply_sign(ev[0][t], sb), apply_sign(ev[W > 1 ? 1 : 0][t], sb));
           } else {
+            red_add_v2(cell, apply_sign(ev[0][t], sb), apply_sign(ev[W > 1 ? 1 : 0][t], sb));
+          }
+          x = step61(x, a);
+          y = step61(y, a2);
+        }
+      }
+    }
+  }
+}
+
+// W >= 4: G = W/4 adjacent lanes share one quad of coordinates; lane `sub` of the group
+// owns workers 4*sub .. 4*sub+3 and, per row and coordinate, issues one 16-byte reduction
+// at offset 4*sub of the cell, so the G lanes of the group cover the whole cell in the same
+// instruction.  The hash is evaluated by every lane of the group (issue slots are not the
+// bound here).
+template <int W, bool ACC, bool VEC, bool POW2>
+__global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_constant__ InsertParams prm) {
+  constexpr int G = W / 4;
+  const int sub = threadIdx.x % G;
+  const int64_t d = prm.d;
+  const int64_t nq = (d + 3) / 4;
+  const int64_t qstride = (int64_t)gridDim.x * (blockDim.x / G);
+  for (int64_t q = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / G; q < nq; q += qstride) {
+    const int64_t i0 = q * 4;
+    float ev[4][4];
 #pragma unroll
-            for (int w4 = 0; w4 < W; w4 += 4) {
-              red_add_v4(cell + w4, apply_sign(ev[w4][t], sb),
-                         apply_sign(ev[w4 + 1 < W ? w4 + 1 : 0][t], sb),
-                         apply_sign(ev[w4 + 2 < W ? w4 + 2 : 0][t], sb),
-                         apply_sign(ev[w4 + 3 < W ? w4 + 3 : 0][t], sb));
-            }
-          }
-          if (t < 3) {
-            x = step61(x, a);
-            y = step61(y, a2);
-          }
+    for (int w4 = 0; w4 < 4; ++w4) {
+      const int w = sub * 4 + w4;
+      if (w < prm.nw) {
+        load_lane<ACC, VEC>(prm, w, i0, d, ev[w4]);
+      } else {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) ev[w4][t] = 0.f;
+      }
+    }
+    const int tmax = (d - i0 < 4) ? (int)(d - i0) : 4;
+#pragma unroll 1
+    for (int j = prm.j0; j < prm.j1; ++j) {
+      const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
+      uint64_t x = affine61(a, prm.h.b[j], (uint32_t)i0);
+      uint64_t y = affine61(a2, prm.h.b2[j], (uint32_t)i0);
+      float* row = prm.table + (size_t)j * prm.c * W + sub * 4;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        if (t < tmax) {
+          const uint32_t bk = bucket_of<POW2>(x, prm.c, prm.cmask);
+          const uint32_t sb = signbit_of(y);
+          red_add_v4(row + (size_t)bk * W, apply_sign(ev[0][t], sb), apply_sign(ev[1][t], sb),
+                     apply_sign(ev[2][t], sb), apply_sign(ev[3][t], sb));
+          x = step61(x, a);
+          y = step61(y, a2);
         }
       }
     }
@@ -156,7 +200,7 @@ __global__ void __launch_bounds__(kBlock) k_insert_lane(const __grid_constant__ 
 #pragma unroll
     for (int t = 0; t < 4; ++t) ev[t] = (t < tmax) ? v[i0 + t] : 0.f;
 #pragma unroll 1
-    for (int j = 0; j < prm.r; ++j) {
+    for (int j = prm.j0; j < prm.j1; ++j) {
       const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
       uint64_t x = affine61(a, prm.h.b[j], (uint32_t)i0);
       uint64_t y = affine61(a2, prm.h.b2[j], (uint32_t)i0);
@@ -204,9 +248,15 @@ int grid_for(K kernel, int64_t work_items, int block) {
 
 template <int W, bool ACC, bool VEC, bool POW2>
 cudaError_t launch_ai_t(const InsertParams& p, cudaStream_t s) {
-  auto kern = k_accumulate_insert<W, ACC, VEC, POW2>;
-  const int grid = grid_for(kern, (p.d + 3) / 4, kBlock);
-  kern<<<grid, kBlock, 0, s>>>(p);
+  if constexpr (W >= 4) {
+    auto kern = k_accumulate_insert_coop<W, ACC, VEC, POW2>;
+    const int grid = grid_for(kern, (p.d + 3) / 4 * (W / 4), kBlock);
+    kern<<<grid, kBlock, 0, s>>>(p);
+  } else {
+    auto kern = k_accumulate_insert<W, ACC, VEC, POW2>;
+    const int grid = grid_for(kern, (p.d + 3) / 4, kBlock);
+    kern<<<grid, kBlock, 0, s>>>(p);
+  }
   return cudaGetLastError();
 }
 
@@ -215,6 +265,11 @@ cudaError_t launch_ai_w(const InsertParams& p, bool vec, cudaStream_t s) {
   const bool pow2 = is_pow2(p.c);
   if (vec) return pow2 ? launch_ai_t<W, ACC, true, true>(p, s) : launch_ai_t<W, ACC, true, false>(p, s);
   return pow2 ? launch_ai_t<W, ACC, false, true>(p, s) : launch_ai_t<W, ACC, false, false>(p, s);
+}
+
+template <int W>
+cudaError_t launch_ai_acc(const InsertParams& p, bool acc, bool vec, cudaStream_t s) {
+  return acc ? launch_ai_w<W, true>(p, vec, s) : launch_ai_w<W, false>(p, vec, s);
 }
 
 }  // namespace
@@ -228,12 +283,12 @@ cudaError_t launch_accumulate(float* u, float* e, const float* g, int64_t d, flo
   return cudaGetLastError();
 }
 
-cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool vec, cudaStream_t s) {
+cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool acc, bool vec, cudaStream_t s) {
   switch (W) {
-    case 1: return launch_ai_w<1, true>(p, vec, s);
-    case 2: return launch_ai_w<2, true>(p, vec, s);
-    case 4: return launch_ai_w<4, true>(p, vec, s);
-    case 8: return launch_ai_w<8, true>(p, vec, s);
+    case 1: return launch_ai_acc<1>(p, acc, vec, s);
+    case 2: return launch_ai_acc<2>(p, acc, vec, s);
+    case 4: return launch_ai_acc<4>(p, acc, vec, s);
+    case 8: return launch_ai_acc<8>(p, acc, vec, s);
     default: return cudaErrorInvalidValue;
   }
 }

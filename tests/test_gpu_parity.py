@@ -109,16 +109,22 @@ def test_single_vector_insert(gs, H, W, worker, P):
         gs.gs_sketch_destroy(sk)
 
 
-@pytest.mark.parametrize("P,W,d,r,c", [(1, 1, 70_001, 3, 1 << 10), (3, 4, 123_457, 5, 1000),
-                                       (5, 8, 200_003, 4, 1 << 13), (8, 2, 65_536, 5, 1 << 12),
-                                       (8, 8, 400_000, 7, 1 << 14), (16, 8, 50_001, 5, 777)])
-def test_accumulate_insert_merge(gs, H, P, W, d, r, c):
+@pytest.mark.parametrize("P,W,d,r,c,passes", [(1, 1, 70_001, 3, 1 << 10, 1), (3, 4, 123_457, 5, 1000, 1),
+                                              (5, 8, 200_003, 4, 1 << 13, 1), (8, 2, 65_536, 5, 1 << 12, 1),
+                                              (8, 8, 400_000, 7, 1 << 14, 1), (16, 8, 50_001, 5, 777, 1),
+                                              (8, 0, 200_003, 3, 1 << 21, 3), (6, 0, 150_001, 5, 1 << 20, 3),
+                                              (4, 0, 100_001, 7, 1 << 21, 4)])
+def test_accumulate_insert_merge(gs, H, P, W, d, r, c, passes):
     seed = P * 1000 + W
     rng = np.random.default_rng(seed)
     coeffs = oracle.derive_coefficients(r, seed)
     run = H.new_run(P, d, r, c, 1, seed, rho=0.9, group_width=W)
     try:
-        assert gs.gs_sketch_info(run.sketch)["group_width"] == W
+        info = gs.gs_sketch_info(run.sketch)
+        if W:
+            assert info["group_width"] == W
+        W = info["group_width"]
+        assert -(-r // info["rows_per_pass"]) == passes
         us = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
         es = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
         gr = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]

@@ -24,4 +24,6 @@ from .gradients import (  # noqa: F401
     spike_positions,
     make_gradient,
     make_gradients,
+    make_gradient_torch,
+    torch_seed,
 )

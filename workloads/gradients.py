@@ -87,3 +87,35 @@ def make_gradients(w: Workload, step: int, workers=None, d: int | None = None, t
     make_gradient(w, step, ws[0], d=1)  # fill the per-config cache before threading
     with ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
         return list(ex.map(lambda p: make_gradient(w, step, p, d=d), ws))
+
+
+def torch_seed(w: Workload, step: int, worker: int) -> int:
+    """64-bit seed of a device-side draw for (workload, step, worker)."""
+    ss = np.random.SeedSequence([BASE_SEED, w.cid, step, worker, 2])
+    return int(ss.generate_state(1, dtype=np.uint64)[0] & np.uint64((1 << 63) - 1))
+
+
+def make_gradient_torch(w: Workload, step: int, worker: int, out):
+    """Fill the fp32 device tensor ``out`` (length d) with a gradient of the same recipe as
+    ``make_gradient``, drawn on the device by PyTorch's generator (a different stream of
+    numbers from the numpy draw, the same distribution).  Used where host generation of
+    hundreds of millions of entries per worker would dominate."""
+    import torch
+    gen = torch.Generator(device=out.device)
+    gen.manual_seed(torch_seed(w, step, worker))
+    if w.dist == "normal":
+        out.normal_(0.0, 1.0, generator=gen)
+    else:
+        out.exponential_(1.0, generator=gen)
+        flip = torch.empty_like(out).uniform_(0.0, 1.0, generator=gen) < 0.5
+        out[flip] = -out[flip]
+        del flip
+    off = 0
+    for size, s in zip(w.blocks, block_scales(w).astype(np.float32)):
+        out[off:off + size].mul_(float(s))
+        off += size
+    pos, sgn = spike_positions(w)
+    if pos.size:
+        pt = torch.from_numpy(pos).to(out.device)
+        out.index_add_(0, pt, torch.from_numpy(sgn * np.float32(w.spike_mag)).to(out.device))
+    return out
