@@ -145,6 +145,28 @@ gs_status gs_query_topk(const gs_sketch* sketch, int64_t d, int64_t k, int64_t* 
                         float* est_out, void* workspace, size_t workspace_bytes,
                         gs_stream stream);
 
+/* Largest d that gs_query_topk_noalloc accepts. */
+#define GS_NOALLOC_MAX_DIM (1LL << 30)
+
+/* gs_query_topk for callers that cannot allocate device memory.  Some hosts hand a library
+ * only the buffers it reads and writes: a framework whose memory pool already holds the
+ * device memory (so a separate cudaMalloc would fail or escape its accounting), an
+ * operator interface with no workspace argument, or a loop that must not pay for the
+ * device-wide synchronisation that cudaMalloc and cudaFree can cause.  This variant
+ * allocates nothing: its scratch (selection histograms, state and per-segment counters,
+ * 1,073,408 bytes) is a fixed array in the library's device memory, which every GPU that
+ * loads the library holds until the process exits.  The paper has no counterpart; this is
+ * a service of the library, not a step of the method.
+ * Same results as gs_query_topk, except that est_out is required (fp32[d], 4-byte aligned)
+ * and d may not exceed GS_NOALLOC_MAX_DIM (larger d returns GS_ERR_INVALID_ARG and
+ * launches nothing).  The first call on a device looks up the scratch array's device
+ * address (a host-side query, no allocation); make that first call before any stream
+ * capture.  Every call on a device shares the one array: each call clears the parts that
+ * must start at zero, and calls whose work overlaps on the GPU (different streams, or
+ * several threads) race on it, so order them on one stream. */
+gs_status gs_query_topk_noalloc(const gs_sketch* sketch, int64_t d, int64_t k, int64_t* idx_out,
+                                float* est_out, gs_stream stream);
+
 /* ---- step 6: second round -------------------------------------------------------- */
 
 /* vals_out[t] = sum over p = 0..P-1 (in that order, fp32) of error[p][idx[t]], then

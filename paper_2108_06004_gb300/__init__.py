@@ -24,6 +24,7 @@ GS_MAX_ROWS = 16
 GS_MAX_COLS = 1 << 26
 GS_MAX_WORKERS = 64
 GS_MAX_DIM = (1 << 31) - 1
+GS_NOALLOC_MAX_DIM = 1 << 30
 
 _lib = None
 
@@ -45,6 +46,7 @@ SIGNATURES = {
     "gs_sketch_merge_tree": [_vp, _i32, _vp],
     "gs_query_topk_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_query_topk": [_vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp],
+    "gs_query_topk_noalloc": [_vp, _i64, _i64, _vp, _vp, _vp],
     "gs_gather_and_zero": [_PP, _PP, _i32, _i64, _vp, _i64, _vp, _vp],
     "gs_step_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_step": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
@@ -173,6 +175,13 @@ def gs_query_topk(sketch: int, d: int, k: int, idx_out, est_out, workspace, work
         workspace_bytes = workspace.numel() * workspace.element_size()
     _check(load_library().gs_query_topk(sketch, d, k, _ptr(idx_out), _ptr(est_out), _ptr(workspace),
                                         workspace_bytes, _stream(stream)), "gs_query_topk")
+
+
+def gs_query_topk_noalloc(sketch: int, d: int, k: int, idx_out, est_out, stream=None) -> None:
+    """gs_query_topk without a caller workspace: the library's fixed device scratch is used
+    (for hosts that cannot allocate device memory; est_out is required)."""
+    _check(load_library().gs_query_topk_noalloc(sketch, d, k, _ptr(idx_out), _ptr(est_out), _stream(stream)),
+           "gs_query_topk_noalloc")
 
 
 def gs_gather_and_zero(momentum, error, d: int, idx, k: int, vals_out, stream=None) -> None:

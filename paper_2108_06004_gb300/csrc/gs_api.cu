@@ -424,6 +424,24 @@ gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_
   return GS_OK;
 }
 
+gs_status gs_query_topk_noalloc(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_out, float* est_out,
+                                gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (d > GS_NOALLOC_MAX_DIM)
+    return fail(GS_ERR_INVALID_ARG, "d = " + std::to_string(d) + " exceeds GS_NOALLOC_MAX_DIM = " +
+                                        std::to_string(GS_NOALLOC_MAX_DIM) +
+                                        ", the size the fixed scratch serves; use gs_query_topk with a workspace");
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  if (!est_out) return fail(GS_ERR_INVALID_ARG, "est_out is required by gs_query_topk_noalloc");
+  GS_TRY(check_vec(est_out, "est_out"));
+  cudaError_t e = gs::launch_query_topk_noalloc(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx_out, est_out,
+                                                as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "query/top-k (no-allocation variant)");
+  return GS_OK;
+}
+
 gs_status gs_gather_and_zero(float* const* momentum, float* const* error, int32_t P, int64_t d, const int64_t* idx,
                              int64_t k, float* vals_out, gs_stream stream) {
   GS_GUARD_BEGIN

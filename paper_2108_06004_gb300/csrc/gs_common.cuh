@@ -122,6 +122,11 @@ size_t query_topk_workspace_bytes(int64_t d, int64_t k);
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
                               void* workspace, cudaStream_t s);
+// Same pipeline with its scratch in a fixed device array (no allocation); est_out required,
+// d <= GS_NOALLOC_MAX_DIM.  The first call on a device looks up the array's address.
+cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, int r, uint32_t c,
+                                      int64_t d, int64_t k, int64_t* idx_out, float* est_out,
+                                      cudaStream_t s);
 
 inline bool is_pow2(uint32_t c) { return c && !(c & (c - 1)); }
 

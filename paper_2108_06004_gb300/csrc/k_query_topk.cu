@@ -15,6 +15,8 @@
 //   k_scan      one CTA: exclusive prefix sums over the segments
 //   k_write     every segment writes its selected indices at their final positions, so the
 //               output is in ascending index order without a sort.
+#include <mutex>
+
 #include "gs_common.cuh"
 
 namespace gs {
@@ -488,6 +490,93 @@ cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, u
   k_scan<<<1, kScanThreads, 0, s>>>(w.blk_gt, w.blk_eq, w.nblk, w.st, w.blk_base, w.blk_eqx);
   if (vec) k_write<true><<<nblk, kBlock, 0, s>>>(est, d, w.st, w.blk_base, w.blk_eqx, idx_out, k);
   else k_write<false><<<nblk, kBlock, 0, s>>>(est, d, w.st, w.blk_base, w.blk_eqx, idx_out, k);
+  return cudaGetLastError();
+}
+
+// ---- scratch without allocation ---------------------------------------------------------
+// For callers that cannot allocate: the selection scratch of the query (three histograms,
+// the state, and four counters per segment of kSeg coordinates, enough for d up to
+// GS_NOALLOC_MAX_DIM) lives in one array of the library's device memory.
+namespace {
+
+constexpr int64_t kNoallocMaxSegs = (GS_NOALLOC_MAX_DIM + kSeg - 1) / kSeg;
+constexpr size_t kNoallocHistBytes = 3 * kBins * sizeof(uint32_t);   // multiple of 256
+constexpr size_t kNoallocStateBytes = 256;
+constexpr size_t kNoallocScratchBytes =
+    kNoallocHistBytes + kNoallocStateBytes + (size_t)kNoallocMaxSegs * 4 * sizeof(uint32_t);
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
+
+// Device address of g_noalloc_scratch on the current device, looked up once per device.
+cudaError_t noalloc_scratch(void** out) {
+  static std::mutex mu;
+  static void* addr[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, int r, uint32_t c,
+                                      int64_t d, int64_t k, int64_t* idx_out, float* est_out,
+                                      cudaStream_t s) {
+  if (d > GS_NOALLOC_MAX_DIM || est_out == nullptr) return cudaErrorInvalidValue;
+  void* base = nullptr;
+  cudaError_t err = noalloc_scratch(&base);
+  if (err != cudaSuccess) return err;
+  char* p = static_cast<char*>(base);
+  uint32_t* hist = reinterpret_cast<uint32_t*>(p);
+  SelectState* st = reinterpret_cast<SelectState*>(p + kNoallocHistBytes);
+  const int64_t nblk = (d + kSeg - 1) / kSeg;
+  uint32_t* blk_gt = reinterpret_cast<uint32_t*>(p + kNoallocHistBytes + kNoallocStateBytes);
+  uint32_t* blk_eq = blk_gt + nblk;
+  uint32_t* blk_base = blk_eq + nblk;
+  uint32_t* blk_eqx = blk_base + nblk;
+  float* est = est_out;
+  const bool vec = (reinterpret_cast<uintptr_t>(est) & 15u) == 0;
+  // the histograms and the state must start at zero; the counters are fully overwritten
+  if ((err = cudaMemsetAsync(hist, 0, kNoallocHistBytes, s)) != cudaSuccess) return err;
+  if ((err = cudaMemsetAsync(st, 0, sizeof(SelectState), s)) != cudaSuccess) return err;
+
+  QueryParams qp;
+  qp.T = merged;
+  qp.est = est;
+  qp.hist = hist;
+  qp.d = d;
+  qp.r = r;
+  qp.c = c;
+  qp.cmask = c - 1;
+  qp.vec = vec ? 1 : 0;
+  qp.h = h;
+  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
+
+  k_pick<<<1, kScanThreads, 0, s>>>(hist, 11, st, 0, (uint32_t)k);
+  const int64_t nq = (d + 3) / 4;
+  const int64_t need = (nq + kBlock - 1) / kBlock;
+  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)k_hist, kBlock);
+  const int hgrid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
+  k_hist<<<hgrid, kBlock, 0, s>>>(est, d, vec ? 1 : 0, st, hist + kBins, 9, 11);
+  k_pick<<<1, kScanThreads, 0, s>>>(hist + kBins, 11, st, 1, 0);
+  k_hist<<<hgrid, kBlock, 0, s>>>(est, d, vec ? 1 : 0, st, hist + 2 * kBins, 0, 9);
+  k_pick<<<1, kScanThreads, 0, s>>>(hist + 2 * kBins, 9, st, 2, 0);
+
+  const int nb = (int)nblk;
+  if (vec) k_count<true><<<nb, kBlock, 0, s>>>(est, d, st, blk_gt, blk_eq);
+  else k_count<false><<<nb, kBlock, 0, s>>>(est, d, st, blk_gt, blk_eq);
+  k_scan<<<1, kScanThreads, 0, s>>>(blk_gt, blk_eq, nblk, st, blk_base, blk_eqx);
+  if (vec) k_write<true><<<nb, kBlock, 0, s>>>(est, d, st, blk_base, blk_eqx, idx_out, k);
+  else k_write<false><<<nb, kBlock, 0, s>>>(est, d, st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();
 }
 
