@@ -65,12 +65,13 @@ typedef void* gs_stream;            /* a cudaStream_t */
  * hash functions), plus the merged r x c table that gs_sketch_merge_tree writes.
  * All tables start at zero.  Worker tables are stored interleaved in groups of
  * `group_width` workers ([group][r][c][group_width] fp32) so that the group's values of a
- * cell are adjacent and are updated by 16-byte vector reductions; group_width 0 lets the
- * library choose (up to 8, no wider than the worker count rounded up to a power of two,
- * halved while one table row exceeds a 64 MiB L2 budget).  The fused insert updates as many
- * rows per pass as fit that budget.
+ * cell are adjacent and are updated by 16-byte vector reductions (G = group_width/4 lanes
+ * together write a whole cell in one instruction); group_width 0 lets the library choose
+ * (up to 16, no wider than the worker count rounded up to a power of two; 16 only when the
+ * whole group table fits a 64 MiB L2 budget, and halved while one table row exceeds it).  The fused insert updates as many rows per pass
+ * as fit that budget.
  * On success *out owns device memory released by gs_sketch_destroy.
- * Errors: GS_ERR_INVALID_ARG (sizes, group_width not in {0,1,2,4,8}, out NULL),
+ * Errors: GS_ERR_INVALID_ARG (sizes, group_width not in {0,1,2,4,8,16}, out NULL),
  *         GS_ERR_OOM (allocation failed), GS_ERR_CUDA.  Synchronous. */
 gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
                            int32_t group_width, gs_sketch** out);
@@ -140,7 +141,13 @@ gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * middle value for odd r, the mean of the two middle values for even r), then the k
  * coordinates of largest |est_i|, ties toward the smaller index, written to idx_out
  * (int64[k]) in ascending order (Alg. 2 steps 1-3).  est_out (fp32[d]) may be NULL.
- * workspace must hold gs_query_topk_workspace_size(d, k) bytes, 256-byte aligned. */
+ * workspace must hold gs_query_topk_workspace_size(d, k) bytes, 256-byte aligned.
+ * When est_out is NULL (and c is a power of two) the query may skip rows: the median of r
+ * values lies between the least and the largest of any floor(r/2)+1 of them, so a
+ * coordinate whose first rows bound |est| below a threshold hint cannot be selected.  The
+ * sketch keeps 0.8 times the previous call's k-th largest |est| as that hint; if the new
+ * threshold turns out below the hint, the query re-runs without skipping, on the device.
+ * The selected indices never depend on the hint. */
 gs_status gs_query_topk(const gs_sketch* sketch, int64_t d, int64_t k, int64_t* idx_out,
                         float* est_out, void* workspace, size_t workspace_bytes,
                         gs_stream stream);
@@ -192,11 +199,15 @@ gs_status gs_step(gs_sketch* sketch, float* const* momentum, float* const* error
                   int64_t* idx_out, float* vals_out, float* est_out, void* workspace,
                   size_t workspace_bytes, gs_stream stream);
 
-/* gs_step with the gradients in HOST memory and the results returned to HOST memory:
- * copies grad_host[p] (pinned host memory gives full copy speed) into the device buffers
- * grad_dev[p], runs gs_step, copies idx (int64[k]) and vals (fp32[k]) back to idx_host
- * and vals_host, and synchronizes `stream` before returning.  Momentum and error stay
- * resident on the device. */
+/* gs_step with the gradients in HOST memory and the results returned to HOST memory, one
+ * synchronous call per step.  Where the device can address grad_host[p] in place (memory
+ * from cudaHostAlloc or cudaHostRegister, or any host memory on systems whose GPU has
+ * pageable-memory access, such as Grace-based GB300 nodes), the fused accumulate+insert
+ * kernel reads it directly over the CPU-GPU link and grad_dev[p] is left unused; otherwise
+ * grad_host[p] is first copied into the device buffer grad_dev[p].  idx (int64[k]) and vals
+ * (fp32[k]) are copied back to idx_host and vals_host, and `stream` is synchronized before
+ * returning.  Momentum and error stay resident on the device.  workspace must hold
+ * gs_step_workspace_size(d, k) bytes. */
 gs_status gs_step_host(gs_sketch* sketch, float* const* momentum, float* const* error,
                        const float* const* grad_host, float* const* grad_dev, int64_t d,
                        float rho, int64_t k, int64_t* idx_host, float* vals_host,

@@ -16,6 +16,7 @@ struct gs_sketch {
   gs::HashCoeffs h;
   float* tables;  // groups * r*c*W
   float* merged;  // r*c
+  uint32_t* hint; // threshold hint of the query (device, one uint32 in a 256-byte slot)
   int device;
 };
 
@@ -62,11 +63,14 @@ void derive_coefficients(int r, uint64_t seed, gs::HashCoeffs& h) {
 // that the table stays resident in the 126 MB L2 while g, u and e stream past it.
 constexpr size_t kL2BudgetBytes = size_t(64) << 20;
 
-// Widest group (up to 8, not wider than the worker count rounded up to a power of two) whose
-// single table row fits the budget.
-int choose_group_width(int c, int workers) {
+// Widest group (up to 16, not wider than the worker count rounded up to a power of two) whose
+// single table row fits the budget.  16-wide groups are used only when the whole group table
+// fits in one pass: their 64-byte cells halve the reduction requests, but a 16-wide table
+// that needs row passes re-reads e more often than two 8-wide groups do (measured slower).
+int choose_group_width(int r, int c, int workers) {
   int W = 1;
   while (W < workers && W < gs::kMaxGroup) W *= 2;
+  if (W == 16 && (size_t)r * (size_t)c * 16 * sizeof(float) > kL2BudgetBytes) W = 8;
   while (W > 1 && (size_t)c * (size_t)W * sizeof(float) > kL2BudgetBytes) W /= 2;
   return W;
 }
@@ -174,7 +178,7 @@ gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float
   mp.group_stride = (int64_t)sk->r * sk->c * sk->W;
   mp.P = sk->workers;
   if ((err = gs::launch_merge(mp, sk->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
-  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, s)) !=
+  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, sk->hint, s)) !=
       cudaSuccess)
     return cuda_fail(err, "query/top-k launch");
   gs::GatherParams gp;
@@ -253,15 +257,17 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   if (r < 1 || r > GS_MAX_ROWS) return fail(GS_ERR_INVALID_ARG, "r must lie in [1, 16]");
   if (c < 1 || c > GS_MAX_COLS) return fail(GS_ERR_INVALID_ARG, "c must lie in [1, 2^26]");
   if (workers < 1 || workers > GS_MAX_WORKERS) return fail(GS_ERR_INVALID_ARG, "workers must lie in [1, 64]");
-  if (group_width != 0 && group_width != 1 && group_width != 2 && group_width != 4 && group_width != 8)
-    return fail(GS_ERR_INVALID_ARG, "group_width must be 0, 1, 2, 4 or 8");
+  if (group_width != 0 && group_width != 1 && group_width != 2 && group_width != 4 && group_width != 8 &&
+      group_width != 16)
+    return fail(GS_ERR_INVALID_ARG, "group_width must be 0, 1, 2, 4, 8 or 16");
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-  const int W = group_width ? group_width : choose_group_width(c, workers);
+  const int W = group_width ? group_width : choose_group_width(r, c, workers);
   const int groups = (workers + W - 1) / W;
   const size_t table_floats = (size_t)groups * r * c * W;
-  const size_t bytes = (table_floats + (size_t)r * c) * sizeof(float);
+  const size_t table_bytes = (table_floats + (size_t)r * c) * sizeof(float);
+  const size_t bytes = ((table_bytes + 255) & ~size_t(255)) + 256;  // + the query's hint slot
   float* mem = nullptr;
   e = cudaMalloc(&mem, bytes);
   if (e != cudaSuccess) {
@@ -285,6 +291,7 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   derive_coefficients(r, seed, sk->h);
   sk->tables = mem;
   sk->merged = mem + table_floats;
+  sk->hint = reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(mem) + ((table_bytes + 255) & ~size_t(255)));
   sk->device = dev;
   *out = sk;
   return ok();
@@ -418,7 +425,7 @@ gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_
   if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
   if (workspace_bytes < gs::query_topk_workspace_bytes(d, k))
     return fail(GS_ERR_INVALID_ARG, "workspace too small: need " + std::to_string(gs::query_topk_workspace_bytes(d, k)));
-  cudaError_t e = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx_out, est_out, workspace,
+  cudaError_t e = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx_out, est_out, workspace, sk->hint,
                                         as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "query/top-k launch");
   return GS_OK;
@@ -512,11 +519,32 @@ gs_status gs_step_host(gs_sketch* sk, float* const* momentum, float* const* erro
   const size_t qbytes = gs::query_topk_workspace_bytes(d, k);
   int64_t* idx_dev = reinterpret_cast<int64_t*>(static_cast<char*>(workspace) + qbytes);
   float* vals_dev = reinterpret_cast<float*>(reinterpret_cast<char*>(idx_dev) + (((size_t)k * 8 + 255) & ~size_t(255)));
+  // Gradients the GPU can address in place (pinned or registered host memory, or any host
+  // memory where the device has pageable-memory access) are read by the fused kernel over
+  // the CPU-GPU link; others are first copied into grad_dev.
+  int pageable = 0;
+  cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, sk->device);
+  std::vector<const float*> gsrc((size_t)sk->workers);
   for (int p = 0; p < sk->workers; ++p) {
-    cudaError_t e = cudaMemcpyAsync(grad_dev[p], grad_host[p], (size_t)d * sizeof(float), cudaMemcpyHostToDevice, s);
-    if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
+    cudaPointerAttributes attr;
+    cudaError_t e = cudaPointerGetAttributes(&attr, grad_host[p]);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      attr.type = cudaMemoryTypeUnregistered;
+    }
+    const float* direct = nullptr;
+    if (attr.type == cudaMemoryTypeHost && attr.devicePointer) direct = static_cast<const float*>(attr.devicePointer);
+    else if (attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged) direct = grad_host[p];
+    else if (attr.type == cudaMemoryTypeUnregistered && pageable == 1) direct = grad_host[p];
+    if (direct && aligned(direct, 4)) {
+      gsrc[(size_t)p] = direct;
+    } else {
+      e = cudaMemcpyAsync(grad_dev[p], grad_host[p], (size_t)d * sizeof(float), cudaMemcpyHostToDevice, s);
+      if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
+      gsrc[(size_t)p] = grad_dev[p];
+    }
   }
-  GS_TRY(step_impl(sk, momentum, error, grad_dev, d, rho, k, idx_dev, vals_dev, nullptr, workspace, s));
+  GS_TRY(step_impl(sk, momentum, error, gsrc.data(), d, rho, k, idx_dev, vals_dev, nullptr, workspace, s));
   cudaError_t e = cudaMemcpyAsync(idx_host, idx_dev, (size_t)k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(vals_host, vals_dev, (size_t)k * sizeof(float), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);

@@ -289,6 +289,7 @@ cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool acc, boo
     case 2: return launch_ai_acc<2>(p, acc, vec, s);
     case 4: return launch_ai_acc<4>(p, acc, vec, s);
     case 8: return launch_ai_acc<8>(p, acc, vec, s);
+    case 16: return launch_ai_acc<16>(p, acc, vec, s);
     default: return cudaErrorInvalidValue;
   }
 }

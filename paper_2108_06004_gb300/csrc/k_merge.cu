@@ -16,7 +16,13 @@ namespace {
 
 template <int W>
 __device__ __forceinline__ void load_group(const float* __restrict__ src, float* v, int lanes) {
-  if (W == 8) {
+  if (W == 16) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 a = __ldcs(reinterpret_cast<const float4*>(src + 4 * q));
+      v[4 * q] = a.x; v[4 * q + 1] = a.y; v[4 * q + 2] = a.z; v[4 * q + 3] = a.w;
+    }
+  } else if (W == 8) {
     const float4 a = __ldcs(reinterpret_cast<const float4*>(src));
     const float4 b = __ldcs(reinterpret_cast<const float4*>(src + 4));
     v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
@@ -91,6 +97,7 @@ cudaError_t launch_merge(const MergeParams& p, int W, cudaStream_t s) {
     case 2: return launch_w<2>(p, s);
     case 4: return launch_w<4>(p, s);
     case 8: return launch_w<8>(p, s);
+    case 16: return launch_w<16>(p, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -90,7 +90,7 @@ def test_accumulate_bit_exact(gs, d, offset):
 
 # ---- step 2 ------------------------------------------------------------------------------
 
-@pytest.mark.parametrize("W,worker,P", [(1, 0, 1), (2, 1, 2), (4, 2, 3), (8, 5, 8), (8, 7, 13)])
+@pytest.mark.parametrize("W,worker,P", [(1, 0, 1), (2, 1, 2), (4, 2, 3), (8, 5, 8), (8, 7, 13), (16, 11, 16)])
 def test_single_vector_insert(gs, H, W, worker, P):
     d, r, c, seed = 300_001, 5, 1 << 12, 5
     rng = np.random.default_rng(W)
@@ -113,7 +113,8 @@ def test_single_vector_insert(gs, H, W, worker, P):
                                               (5, 8, 200_003, 4, 1 << 13, 1), (8, 2, 65_536, 5, 1 << 12, 1),
                                               (8, 8, 400_000, 7, 1 << 14, 1), (16, 8, 50_001, 5, 777, 1),
                                               (8, 0, 200_003, 3, 1 << 21, 3), (6, 0, 150_001, 5, 1 << 20, 3),
-                                              (4, 0, 100_001, 7, 1 << 21, 4)])
+                                              (4, 0, 100_001, 7, 1 << 21, 4), (16, 16, 90_001, 5, 1 << 12, 1),
+                                              (13, 0, 80_003, 3, 1 << 20, 2), (16, 0, 70_001, 5, 1 << 16, 1), (20, 16, 60_001, 4, 3001, 1)])
 def test_accumulate_insert_merge(gs, H, P, W, d, r, c, passes):
     seed = P * 1000 + W
     rng = np.random.default_rng(seed)
@@ -278,3 +279,74 @@ def test_steps_ragged(gs, H, P, r, c, k, W):
 def test_steps_resnet18_full_size(gs, H):
     w = workloads.get_config("resnet18")
     _run_steps(gs, H, w, w.d, 2)
+
+
+@pytest.mark.parametrize("kind", ["pinned", "pageable", "device"])
+def test_step_host_buffers(gs, H, kind):
+    """gs_step_host with gradients in pinned host memory, in plain (pageable) numpy arrays and
+    in device memory; results returned to host buffers."""
+    w = workloads.get_config("resnet18")
+    P, d, r, c, k, seed = 5, 300_001, 5, 4096, 300, 41
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho)
+    try:
+        gdev_buf = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+        idx_h = torch.empty(k, dtype=torch.int64).pin_memory()
+        vals_h = torch.empty(k, dtype=torch.float32).pin_memory()
+        for t in range(2):
+            grads = workloads.make_gradients(w, t, range(P), d=d)
+            if kind == "pinned":
+                src = [torch.from_numpy(g).pin_memory() for g in grads]
+            elif kind == "pageable":
+                src = [np.ascontiguousarray(g) for g in grads]
+            else:
+                src = [_dev(g) for g in grads]
+            ptrs = [s.ctypes.data if isinstance(s, np.ndarray) else s for s in src]
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            gs.gs_step_host(run.sketch, run.us, run.es, ptrs, gdev_buf, d, w.rho, k, idx_h, vals_h, run.ws)
+            res = oracle.step(us0, es0, grads, w.rho, coeffs, c, k)
+            idx = idx_h.numpy().copy()
+            band = oracle.cell_band(res.merged_abs, coeffs, np.arange(d))
+            H.check_topk_set(idx, res.idx, res.est, band, k, d)
+            H.check_state([H.host(u) for u in run.us], [H.host(e) for e in run.es], res, idx)
+            H.check_vals(vals_h.numpy().copy(), idx, res.es_pre)
+    finally:
+        run.close()
+
+
+@pytest.mark.parametrize("r", [5, 4, 7])
+def test_pruned_query_matches_exact(gs, H, r):
+    """With est_out = NULL the query may skip rows against the previous call's threshold
+    hint; the selection must equal the unpruned query's on the same merged table and agree
+    with the oracle -- also when the threshold collapses below the hint (exact re-run)."""
+    w = workloads.get_config("resnet18")
+    P, d, c, k, seed = 4, 400_003, 1 << 13, 500, 91
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho)
+    try:
+        ws_q = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        idx_exact = torch.empty(k, dtype=torch.int64, device="cuda")
+        for t in range(5):
+            grads = workloads.make_gradients(w, t, range(P), d=d)
+            if t == 3:  # collapse the state and the gradients: the threshold falls far below the hint
+                for u, e in zip(run.us, run.es):
+                    u.zero_()
+                    e.zero_()
+                grads = [(g * np.float32(1e-3)).astype(np.float32) for g in grads]
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            gs.gs_step(run.sketch, run.us, run.es, [_dev(g) for g in grads], d, w.rho, k, run.idx, run.vals,
+                       None, run.ws)
+            gs.gs_query_topk(run.sketch, d, k, idx_exact, run.est, ws_q)   # unpruned, same merged table
+            torch.cuda.synchronize()
+            idx = H.host(run.idx)
+            assert np.array_equal(idx, H.host(idx_exact)), f"step {t}: pruned selection differs"
+            H.check_selection_exact(idx, H.host(run.est), k)
+            res = oracle.step(us0, es0, grads, w.rho, coeffs, c, k)
+            band = oracle.cell_band(res.merged_abs, coeffs, np.arange(d))
+            H.check_topk_set(idx, res.idx, res.est, band, k, d)
+            H.check_state([H.host(u) for u in run.us], [H.host(e) for e in run.es], res, idx)
+            H.check_vals(H.host(run.vals), idx, res.es_pre)
+    finally:
+        run.close()
