@@ -141,13 +141,9 @@ gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * middle value for odd r, the mean of the two middle values for even r), then the k
  * coordinates of largest |est_i|, ties toward the smaller index, written to idx_out
  * (int64[k]) in ascending order (Alg. 2 steps 1-3).  est_out (fp32[d]) may be NULL.
- * workspace must hold gs_query_topk_workspace_size(d, k) bytes, 256-byte aligned.
- * When est_out is NULL (and c is a power of two) the query may skip rows: the median of r
- * values lies between the least and the largest of any floor(r/2)+1 of them, so a
- * coordinate whose first rows bound |est| below a threshold hint cannot be selected.  The
- * sketch keeps 0.8 times the previous call's k-th largest |est| as that hint; if the new
- * threshold turns out below the hint, the query re-runs without skipping, on the device.
- * The selected indices never depend on the hint. */
+ * workspace must hold gs_query_topk_workspace_size(d, k) bytes, 256-byte aligned (about
+ * 12.3 bytes per coordinate: the estimate, room for a candidate list of (index, key) pairs,
+ * and two d-bit bitmaps). */
 gs_status gs_query_topk(const gs_sketch* sketch, int64_t d, int64_t k, int64_t* idx_out,
                         float* est_out, void* workspace, size_t workspace_bytes,
                         gs_stream stream);

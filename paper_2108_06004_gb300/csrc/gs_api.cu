@@ -16,7 +16,6 @@ struct gs_sketch {
   gs::HashCoeffs h;
   float* tables;  // groups * r*c*W
   float* merged;  // r*c
-  uint32_t* hint; // threshold hint of the query (device, one uint32 in a 256-byte slot)
   int device;
 };
 
@@ -178,7 +177,7 @@ gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float
   mp.group_stride = (int64_t)sk->r * sk->c * sk->W;
   mp.P = sk->workers;
   if ((err = gs::launch_merge(mp, sk->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
-  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, sk->hint, s)) !=
+  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, s)) !=
       cudaSuccess)
     return cuda_fail(err, "query/top-k launch");
   gs::GatherParams gp;
@@ -266,8 +265,7 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   const int W = group_width ? group_width : choose_group_width(r, c, workers);
   const int groups = (workers + W - 1) / W;
   const size_t table_floats = (size_t)groups * r * c * W;
-  const size_t table_bytes = (table_floats + (size_t)r * c) * sizeof(float);
-  const size_t bytes = ((table_bytes + 255) & ~size_t(255)) + 256;  // + the query's hint slot
+  const size_t bytes = (table_floats + (size_t)r * c) * sizeof(float);
   float* mem = nullptr;
   e = cudaMalloc(&mem, bytes);
   if (e != cudaSuccess) {
@@ -291,7 +289,6 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   derive_coefficients(r, seed, sk->h);
   sk->tables = mem;
   sk->merged = mem + table_floats;
-  sk->hint = reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(mem) + ((table_bytes + 255) & ~size_t(255)));
   sk->device = dev;
   *out = sk;
   return ok();
@@ -425,7 +422,7 @@ gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_
   if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
   if (workspace_bytes < gs::query_topk_workspace_bytes(d, k))
     return fail(GS_ERR_INVALID_ARG, "workspace too small: need " + std::to_string(gs::query_topk_workspace_bytes(d, k)));
-  cudaError_t e = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx_out, est_out, workspace, sk->hint,
+  cudaError_t e = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx_out, est_out, workspace,
                                         as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "query/top-k launch");
   return GS_OK;

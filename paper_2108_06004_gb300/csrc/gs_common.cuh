@@ -119,11 +119,9 @@ cudaError_t launch_merge(const MergeParams& p, int W, cudaStream_t s);
 cudaError_t launch_gather_and_zero(const GatherParams& p, cudaStream_t s);
 
 size_t query_topk_workspace_bytes(int64_t d, int64_t k);
-// hint: the sketch's threshold-hint slot (device uint32, nullable); used only when est_out is
-// NULL, to skip rows of coordinates that provably stay below the previous threshold.
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, uint32_t* hint, cudaStream_t s);
+                              void* workspace, cudaStream_t s);
 // Same pipeline with its scratch in a fixed device array (no allocation); est_out required,
 // d <= GS_NOALLOC_MAX_DIM.  The first call on a device looks up the array's address.
 cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, int r, uint32_t c,

@@ -1,21 +1,26 @@
 // Steps 4 and 5: median-of-r query of the merged sketch and top-k selection
 // (Alg. 2 steps 1-3, read as a deterministic top-k by |est| with ties to the smaller index).
 //
-// Pipeline (all on one stream, no host round trip):
-//   k_query     est_i = median_j s_j(i) T[j][h_j(i)] for every i, written as fp32, and a
-//               2048-bin histogram of key bits 30..20, key = bits of |est_i| (for
-//               non-negative floats the bit pattern orders like the value).
-//   k_hist      histogram of the next key bits among keys in the chosen bin (bits 19..9,
-//               then bits 8..0).
-//               Each of these kernels ends with a pick: the last CTA to finish (found with a
-//               counter after a memory fence, so no CTA waits for another) finds the bin that
-//               holds the k-th largest key and how many keys of that bin are still to be
-//               taken.  After three levels the k-th largest key tau is exact, and
-//               need_eq = k - #{key > tau} keys equal to tau are taken, those of smallest index.
-//   k_count     per segment of 16384 coordinates: #{key > tau}, #{key == tau}
-//   k_scan      one CTA: exclusive prefix sums over the segments
-//   k_write     every segment writes its selected indices at their final positions, so the
-//               output is in ascending index order without a sort.
+// The selection is a radix select on key = bits of |est| (for non-negative floats the bit
+// pattern orders like the value) in three levels: bits 30..20, 19..9 and 8..0.  Each
+// histogram kernel ends with a pick: the last CTA to finish (found with a counter after a
+// memory fence, so no CTA waits for another) finds the bin that holds the k-th largest key
+// and how many keys of that bin are still to be taken.  After three levels the k-th largest
+// key tau is exact, and need_eq = k - #{key > tau} keys equal to tau are taken, those of
+// smallest index.  Output indices are ascending.
+//
+// With a caller workspace (gs_query_topk):
+//   k_query       est_i for every i (fp32) + level-1 histogram + pick
+//   k_cand        one pass over est: keys above the picked level-1 bin are selected for
+//                 certain and set their bit in a d-bit bitmap; keys inside the bin become
+//                 candidates (index, key) and feed the level-2 histogram + pick
+//   k_cand_hist3  level-3 histogram of the candidates + pick
+//   k_cand_mark   candidates above tau into the bitmap, candidates equal to tau into a second
+//   k_bm_count    per block of 65536 coordinates: bits set in each bitmap
+//   k_scan        one CTA: exclusive prefix sums over the blocks
+//   k_bm_write    every block writes its selected indices at their final positions
+// With the fixed scratch (gs_query_topk_noalloc), which cannot hold candidate lists, the
+// levels 2 and 3 and the final selection read est in full passes (k_hist, k_count, k_write).
 #include <mutex>
 
 #include "gs_common.cuh"
@@ -25,11 +30,9 @@ namespace gs {
 namespace {
 
 constexpr int kBins = 2048;
-constexpr int kSegThreads = 256;
-constexpr int kPerThread = 64;                      // consecutive coordinates per thread
-constexpr int kSeg = kSegThreads * kPerThread;      // 16384 coordinates per segment
 constexpr int kScanThreads = 1024;
 constexpr uint32_t kNone = 0xFFFFFFFFu;
+constexpr uint32_t kFull = 0xFFFFFFFFu;
 
 struct SelectState {
   uint32_t prefix;   // key bits fixed so far
@@ -37,46 +40,17 @@ struct SelectState {
   uint32_t tau;      // the k-th largest key
   uint32_t need_eq;  // keys equal to tau to take
   uint32_t found;    // bit l set when level l found its bin
-  uint32_t fail;     // pruned query: the threshold fell below the hint (result not usable)
+  uint32_t ncand;    // candidates appended by k_cand
   uint32_t done[3];  // CTAs finished per level (for the last-CTA pick)
 };
 
-struct Workspace {
-  float* est;
-  uint32_t* hist;     // 6 * kBins: three levels for the first pass, three for the exact re-run
-  SelectState* st;    // two states: first pass, exact re-run
-  uint32_t* blk_gt;   // nblk each
-  uint32_t* blk_eq;
-  uint32_t* blk_base;
-  uint32_t* blk_eqx;
-  int64_t nblk;
-};
-
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
-
-Workspace carve(void* base, int64_t d) {
-  Workspace w;
-  char* p = static_cast<char*>(base);
-  const int64_t nblk = (d + kSeg - 1) / kSeg;
-  w.est = reinterpret_cast<float*>(p);
-  p += align256((size_t)d * sizeof(float));
-  w.hist = reinterpret_cast<uint32_t*>(p);
-  p += align256(6 * kBins * sizeof(uint32_t));
-  w.st = reinterpret_cast<SelectState*>(p);
-  p += 2 * align256(sizeof(SelectState));
-  w.blk_gt = reinterpret_cast<uint32_t*>(p);
-  w.blk_eq = w.blk_gt + nblk;
-  w.blk_base = w.blk_eq + nblk;
-  w.blk_eqx = w.blk_base + nblk;
-  w.nblk = nblk;
-  return w;
-}
 
 __device__ __forceinline__ uint32_t key_of(float v) { return __float_as_uint(v) & 0x7FFFFFFFu; }
 
 // Warp-aggregated shared-memory histogram update; every lane of the warp must call it.
 __device__ __forceinline__ void hist_add(uint32_t* sh, uint32_t bin) {
-  const uint32_t peers = __match_any_sync(0xFFFFFFFFu, bin);
+  const uint32_t peers = __match_any_sync(kFull, bin);
   const int leader = __ffs(peers) - 1;
   if (bin != kNone && (int)(threadIdx.x & 31) == leader) atomicAdd(&sh[bin], (uint32_t)__popc(peers));
 }
@@ -97,7 +71,7 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* total)
   uint32_t x = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+    const uint32_t y = __shfl_up_sync(kFull, x, o);
     if (lane >= o) x += y;
   }
   if (lane == 31) warp_sums[warp] = x;
@@ -106,7 +80,7 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* total)
     uint32_t w = lane < nwarps ? warp_sums[lane] : 0u;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, w, o);
+      const uint32_t y = __shfl_up_sync(kFull, w, o);
       if (lane >= o) w += y;
     }
     warp_sums[lane] = w;
@@ -118,13 +92,19 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* total)
   return off + x - v;
 }
 
+__device__ __forceinline__ uint32_t warp_incl_scan(uint32_t x) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFull, x, o);
+    if (lane >= o) x += y;
+  }
+  return x;
+}
+
 // The whole block finds the bin holding the k_rem-th largest key, scanning from the top bin.
 // Histogram values are read past L1 (they were completed by other CTAs' atomics).
-// At the last level, with a hint slot: `check` records whether the threshold reached the hint
-// the pruned query used (else its result is not usable), and the slot gets the hint for the
-// next query, 0.8 times this threshold.
-__device__ void pick_bins(const uint32_t* hist, int nbits, SelectState* st, int level, uint32_t k_init,
-                          uint32_t* hint, int check) {
+__device__ void pick_bins(const uint32_t* hist, int nbits, SelectState* st, int level, uint32_t k_init) {
   const int nbins = 1 << nbits;
   const uint32_t k_rem = level == 0 ? k_init : __ldcg(&st->k_rem);
   const uint32_t prefix = level == 0 ? 0u : __ldcg(&st->prefix);
@@ -151,11 +131,6 @@ __device__ void pick_bins(const uint32_t* hist, int nbits, SelectState* st, int 
       if (level == 2) {
         st->tau = p;
         st->need_eq = k_rem - cum;
-        if (hint) {
-          const uint32_t used = __ldcg(hint);
-          if (check) st->fail = (p < used) ? 1u : 0u;
-          *hint = key_of(0.8f * __uint_as_float(p));
-        }
       }
     }
     cum += cnt;
@@ -164,7 +139,7 @@ __device__ void pick_bins(const uint32_t* hist, int nbits, SelectState* st, int 
 
 // Called by every CTA after its histogram atomics: the last CTA to arrive does the pick.
 __device__ __forceinline__ void last_block_pick(const uint32_t* hist, int nbits, SelectState* st, int level,
-                                                uint32_t k_init, uint32_t* hint = nullptr, int check = 0) {
+                                                uint32_t k_init) {
   __shared__ uint32_t am_last;
   __threadfence();
   __syncthreads();
@@ -172,7 +147,7 @@ __device__ __forceinline__ void last_block_pick(const uint32_t* hist, int nbits,
   __syncthreads();
   if (am_last) {
     __threadfence();
-    pick_bins(hist, nbits, st, level, k_init, hint, check);
+    pick_bins(hist, nbits, st, level, k_init);
   }
 }
 
@@ -201,8 +176,6 @@ struct QueryParams {
   int32_t r;
   uint32_t c, cmask;
   int32_t vec;        // est 16-byte aligned
-  const uint32_t* gate;  // exact re-run: run only if *gate (the first pass's fail flag) is set
-  const uint32_t* hint;  // pruned query: hint key (read once)
   HashCoeffs h;
 };
 
@@ -215,19 +188,15 @@ __device__ __forceinline__ void store_est(const QueryParams& prm, int64_t i0, in
   }
 }
 
-// Fast path: R rows known at compile time, c a power of two.
-// PRUNE: read the first M = R/2 + 1 rows; the median of all R values lies between the least
-// and the largest of any M of them, so |est| <= max_j<M |v_j|.  When that bound is below the
-// hint key the coordinate cannot reach the threshold the hint stands for; its remaining rows
-// are skipped and 0 is stored (the last pick checks that the threshold did reach the hint).
-template <int R, bool PRUNE>
+// ---- the query ----------------------------------------------------------------------------
+
+// Fast path: R rows known at compile time, c a power of two.  A thread takes four consecutive
+// coordinates; their hash values after the first come from the incremental form.
+template <int R>
 __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryParams prm) {
-  if (prm.gate && __ldcg(prm.gate) == 0u) return;  // uniform: the exact re-run is not needed
-  constexpr int M = PRUNE ? R / 2 + 1 : R;
   __shared__ uint32_t sh[kBins];
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
   __syncthreads();
-  const uint32_t hk = PRUNE ? __ldcg(prm.hint) : 0u;
   const int64_t d = prm.d, nq = (d + 3) / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int lane = threadIdx.x & 31;
@@ -239,7 +208,7 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
     if (tmax > 0) {
       float v[4][R];
 #pragma unroll
-      for (int j = 0; j < M; ++j) {
+      for (int j = 0; j < R; ++j) {
         uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
         uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
         const float* row = prm.T + (size_t)j * prm.c;
@@ -253,33 +222,8 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
           }
         }
       }
-      bool need[4];
 #pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        float ub = 0.f;
-#pragma unroll
-        for (int j = 0; j < M; ++j) ub = fmaxf(ub, fabsf(v[t][j]));
-        need[t] = t < tmax && (!PRUNE || key_of(ub) >= hk);
-      }
-      if (PRUNE && (need[0] || need[1] || need[2] || need[3])) {
-#pragma unroll
-        for (int j = M; j < R; ++j) {
-          uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
-          uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
-          const float* row = prm.T + (size_t)j * prm.c;
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            v[t][j] = 0.f;
-            if (t < tmax) {
-              if (need[t]) v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
-              x = step61(x, prm.h.a[j]);
-              y = step61(y, prm.h.a2[j]);
-            }
-          }
-        }
-      }
-#pragma unroll
-      for (int t = 0; t < 4; ++t) m[t] = need[t] ? median_of<R>(v[t]) : 0.f;
+      for (int t = 0; t < 4; ++t) m[t] = median_of<R>(v[t]);
       store_est(prm, i0, tmax, m);
     }
 #pragma unroll
@@ -291,7 +235,6 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
 
 // General path: any r <= 16 and any c (bucket by 64-bit remainder).
 __global__ void __launch_bounds__(kBlock) k_query_generic(const __grid_constant__ QueryParams prm) {
-  if (prm.gate && __ldcg(prm.gate) == 0u) return;
   __shared__ uint32_t sh[kBins];
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
   __syncthreads();
@@ -329,14 +272,226 @@ __global__ void __launch_bounds__(kBlock) k_query_generic(const __grid_constant_
   last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
 }
 
+// Four float4 of est per thread in flight (kU strides of the grid-stride loop).
+constexpr int kU = 4;
+
+__device__ __forceinline__ void load_quads(const float* __restrict__ est, int64_t d, int vec, int64_t q0,
+                                           int64_t stride, float (&v)[kU][4], int (&tm)[kU]) {
+  const int64_t nq = (d + 3) / 4;
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int u = 0; u < kU; ++u) {
+    const int64_t q = q0 + u * stride + lane;
+    const int64_t i0 = q * 4;
+    tm[u] = q < nq ? (d - i0 < 4 ? (int)(d - i0) : 4) : 0;
+    if (vec && tm[u] == 4) {
+      const float4 f = __ldcs(reinterpret_cast<const float4*>(est + i0));
+      v[u][0] = f.x; v[u][1] = f.y; v[u][2] = f.z; v[u][3] = f.w;
+    } else {
+#pragma unroll
+      for (int t = 0; t < 4; ++t) v[u][t] = t < tm[u] ? est[i0 + t] : 0.f;
+    }
+  }
+}
+
+// ---- selection with candidate lists --------------------------------------------------------
+
+// One pass over est after the level-1 pick.  Keys above the level-1 bin are selected for
+// certain: their bit goes into gt_bm.  Keys inside the bin are appended to `cand` (index, key)
+// and feed the level-2 histogram; the level-2 pick follows.  A warp reserves room for all
+// candidates of its kU x 4 slots with a single atomic on the shared counter.
+__global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ est, int64_t d, int vec,
+                                                 SelectState* st, uint32_t* hist2, uint2* __restrict__ cand,
+                                                 uint32_t* gt_bm) {
+  __shared__ uint32_t sh[kBins];
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
+  __syncthreads();
+  const uint32_t b1 = __ldcg(&st->prefix);
+  const int64_t nq = (d + 3) / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int lane = threadIdx.x & 31;
+  const uint32_t lower = (1u << lane) - 1u;
+  for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += kU * stride) {
+    float v[kU][4];
+    int tm[kU];
+    load_quads(est, d, vec, q0, stride, v, tm);
+    uint32_t keys[kU][4];
+    uint32_t slot_mask[kU][4];
+    uint32_t total = 0;
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t i0 = (q0 + u * stride + lane) * 4;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const uint32_t key = key_of(v[u][t]);
+        const bool valid = t < tm[u];
+        const uint32_t bin1 = key >> 20;
+        const int64_t i = i0 + t;
+        if (valid && bin1 > b1) atomicOr(&gt_bm[i >> 5], 1u << (i & 31));
+        keys[u][t] = key;
+        slot_mask[u][t] = __ballot_sync(kFull, valid && bin1 == b1);
+        total += __popc(slot_mask[u][t]);
+      }
+    }
+    if (total == 0) continue;  // warp-uniform
+    uint32_t base = 0;
+    if (lane == 0) base = atomicAdd(&st->ncand, total);
+    base = __shfl_sync(kFull, base, 0);
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t i0 = (q0 + u * stride + lane) * 4;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const uint32_t m = slot_mask[u][t];
+        if (m) {
+          const bool in = (m >> lane) & 1u;
+          if (in) cand[base + __popc(m & lower)] = make_uint2((uint32_t)(i0 + t), keys[u][t]);
+          hist_add(sh, in ? ((keys[u][t] >> 9) & (kBins - 1)) : kNone);
+          base += __popc(m);
+        }
+      }
+    }
+  }
+  hist_flush(sh, hist2, kBins);
+  last_block_pick(hist2, 11, st, 1, 0);
+}
+
+// Level-3 histogram of the candidates that match the 22-bit prefix; the last pick gives tau.
+__global__ void __launch_bounds__(kBlock) k_cand_hist3(const uint2* __restrict__ cand, SelectState* st,
+                                                       uint32_t* hist3) {
+  __shared__ uint32_t sh[512];
+  for (int b = threadIdx.x; b < 512; b += blockDim.x) sh[b] = 0;
+  __syncthreads();
+  const uint32_t n = __ldcg(&st->ncand);
+  const uint32_t p22 = __ldcg(&st->prefix);
+  const uint32_t stride = gridDim.x * blockDim.x;
+  const int lane = threadIdx.x & 31;
+  for (uint32_t t0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); t0 < n; t0 += stride) {
+    const uint32_t t = t0 + lane;
+    uint32_t bin = kNone;
+    if (t < n) {
+      const uint32_t key = cand[t].y;
+      if ((key >> 9) == p22) bin = key & 511u;
+    }
+    if (__any_sync(kFull, bin != kNone)) hist_add(sh, bin);
+  }
+  hist_flush(sh, hist3, 512);
+  last_block_pick(hist3, 9, st, 2, 0);
+}
+
+// Candidates above tau into gt_bm, candidates equal to tau into eq_bm.
+__global__ void __launch_bounds__(kBlock) k_cand_mark(const uint2* __restrict__ cand, const SelectState* st,
+                                                      uint32_t* gt_bm, uint32_t* eq_bm) {
+  const uint32_t n = __ldcg(&st->ncand);
+  const uint32_t tau = __ldcg(&st->tau);
+  for (uint32_t t = blockIdx.x * blockDim.x + threadIdx.x; t < n; t += gridDim.x * blockDim.x) {
+    const uint2 c = cand[t];
+    if (c.y > tau) atomicOr(&gt_bm[c.x >> 5], 1u << (c.x & 31));
+    else if (c.y == tau) atomicOr(&eq_bm[c.x >> 5], 1u << (c.x & 31));
+  }
+}
+
+constexpr int kBmThreads = 256;
+constexpr int kBmWordsPerThread = 8;
+constexpr int kBmWords = kBmThreads * kBmWordsPerThread;  // 2048 words = 65536 coordinates per block
+
+__global__ void __launch_bounds__(kBmThreads) k_bm_count(const uint32_t* __restrict__ gt_bm,
+                                                         const uint32_t* __restrict__ eq_bm, int64_t nbw,
+                                                         uint32_t* blk_gt, uint32_t* blk_eq) {
+  const int64_t w0 = (int64_t)blockIdx.x * kBmWords + (int64_t)threadIdx.x * kBmWordsPerThread;
+  uint32_t gt = 0, eq = 0;
+#pragma unroll
+  for (int j = 0; j < kBmWordsPerThread; ++j) {
+    if (w0 + j < nbw) {
+      gt += __popc(__ldcg(&gt_bm[w0 + j]));
+      eq += __popc(__ldcg(&eq_bm[w0 + j]));
+    }
+  }
+  uint32_t tg, te;
+  block_excl_scan(gt, &tg);
+  block_excl_scan(eq, &te);
+  if (threadIdx.x == 0) {
+    blk_gt[blockIdx.x] = tg;
+    blk_eq[blockIdx.x] = te;
+  }
+}
+
+__global__ void __launch_bounds__(kScanThreads) k_scan(const uint32_t* __restrict__ blk_gt,
+                                                       const uint32_t* __restrict__ blk_eq, int64_t nblk,
+                                                       const SelectState* st, uint32_t* blk_base,
+                                                       uint32_t* blk_eqx) {
+  const uint32_t need_eq = __ldcg(&st->need_eq);
+  uint32_t carry_gt = 0, carry_eq = 0;
+  for (int64_t c0 = 0; c0 < nblk; c0 += blockDim.x) {
+    const int64_t b = c0 + threadIdx.x;
+    const uint32_t g = b < nblk ? blk_gt[b] : 0u;
+    const uint32_t e = b < nblk ? blk_eq[b] : 0u;
+    uint32_t tg, te;
+    const uint32_t xg = block_excl_scan(g, &tg) + carry_gt;
+    const uint32_t xe = block_excl_scan(e, &te) + carry_eq;
+    if (b < nblk) {
+      blk_base[b] = xg + (xe < need_eq ? xe : need_eq);
+      blk_eqx[b] = xe;
+    }
+    carry_gt += tg;
+    carry_eq += te;
+  }
+}
+
+// Walks the set bits of each thread's words in index order: bits of gt_bm are taken, bits of
+// eq_bm are taken while their rank among the keys equal to tau is below need_eq.
+__global__ void __launch_bounds__(kBmThreads) k_bm_write(const uint32_t* __restrict__ gt_bm,
+                                                         const uint32_t* __restrict__ eq_bm, int64_t nbw,
+                                                         const SelectState* st, const uint32_t* __restrict__ blk_base,
+                                                         const uint32_t* __restrict__ blk_eqx,
+                                                         int64_t* __restrict__ idx_out, int64_t k) {
+  const uint32_t need_eq = __ldcg(&st->need_eq);
+  const uint32_t base = blk_base[blockIdx.x];
+  const uint32_t eqx = blk_eqx[blockIdx.x];
+  const int64_t w0 = (int64_t)blockIdx.x * kBmWords + (int64_t)threadIdx.x * kBmWordsPerThread;
+  uint32_t g[kBmWordsPerThread], e[kBmWordsPerThread];
+  uint32_t gt = 0, eq = 0;
+#pragma unroll
+  for (int j = 0; j < kBmWordsPerThread; ++j) {
+    const bool in = w0 + j < nbw;
+    g[j] = in ? __ldcg(&gt_bm[w0 + j]) : 0u;
+    e[j] = in ? __ldcg(&eq_bm[w0 + j]) : 0u;
+    gt += __popc(g[j]);
+    eq += __popc(e[j]);
+  }
+  uint32_t tg, te;
+  const uint32_t pre_gt = block_excl_scan(gt, &tg);
+  const uint32_t pre_eq = block_excl_scan(eq, &te);
+  if (gt + eq == 0) return;
+  const uint32_t eq_quota = need_eq > eqx ? need_eq - eqx : 0u;  // this block's share of ties
+  uint32_t pos = base + pre_gt + (pre_eq < eq_quota ? pre_eq : eq_quota);
+  uint32_t eq_rank = pre_eq;
+#pragma unroll
+  for (int j = 0; j < kBmWordsPerThread; ++j) {
+    uint32_t bits = g[j] | e[j];
+    while (bits) {
+      const int b = __ffs(bits) - 1;
+      bits &= bits - 1u;
+      bool take = (g[j] >> b) & 1u;
+      if (!take) {
+        take = eq_rank < eq_quota;
+        ++eq_rank;
+      }
+      if (take) {
+        if ((int64_t)pos < k) idx_out[pos] = (w0 + j) * 32 + b;
+        ++pos;
+      }
+    }
+  }
+}
+
+// ---- selection by full passes over est (fixed-scratch variant) -----------------------------
+
 // Histogram of key bits [shift, shift + nbits) among keys whose bits above are the prefix
-// picked at the previous level; ends with the pick of this level.  Each thread loads four
-// float4 before it processes them, to keep enough L2 reads in flight.
+// picked at the previous level; ends with the pick of this level.
 __global__ void __launch_bounds__(kBlock) k_hist(const float* __restrict__ est, int64_t d, int vec,
                                                  SelectState* st, uint32_t* hist, int shift, int nbits,
-                                                 int level, const uint32_t* gate, uint32_t* hint, int check) {
-  if (gate && __ldcg(gate) == 0u) return;  // uniform: the exact re-run is not needed
-  constexpr int U = 4;
+                                                 int level) {
   __shared__ uint32_t sh[kBins];
   const int nbins = 1 << nbits;
   for (int b = threadIdx.x; b < nbins; b += blockDim.x) sh[b] = 0;
@@ -345,25 +500,12 @@ __global__ void __launch_bounds__(kBlock) k_hist(const float* __restrict__ est, 
   const int match_shift = shift + nbits;
   const int64_t nq = (d + 3) / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  const int lane = threadIdx.x & 31;
-  for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += U * stride) {
-    float v[U][4];
-    int tm[U];
+  for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += kU * stride) {
+    float v[kU][4];
+    int tm[kU];
+    load_quads(est, d, vec, q0, stride, v, tm);
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int64_t q = q0 + u * stride + lane;
-      const int64_t i0 = q * 4;
-      tm[u] = q < nq ? (d - i0 < 4 ? (int)(d - i0) : 4) : 0;
-      if (vec && tm[u] == 4) {
-        const float4 f = __ldcs(reinterpret_cast<const float4*>(est + i0));
-        v[u][0] = f.x; v[u][1] = f.y; v[u][2] = f.z; v[u][3] = f.w;
-      } else {
-#pragma unroll
-        for (int t = 0; t < 4; ++t) v[u][t] = t < tm[u] ? est[i0 + t] : 0.f;
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
+    for (int u = 0; u < kU; ++u) {
       uint32_t bins[4];
       bool any = false;
 #pragma unroll
@@ -373,19 +515,21 @@ __global__ void __launch_bounds__(kBlock) k_hist(const float* __restrict__ est, 
         bins[t] = hit ? ((key >> shift) & (uint32_t)(nbins - 1)) : kNone;
         any = any || hit;
       }
-      if (__any_sync(0xFFFFFFFFu, any)) {  // most warps hold no key of the chosen bin
+      if (__any_sync(kFull, any)) {  // most warps hold no key of the chosen bin
 #pragma unroll
         for (int t = 0; t < 4; ++t) hist_add(sh, bins[t]);
       }
     }
   }
   hist_flush(sh, hist, nbins);
-  last_block_pick(hist, nbits, st, level, 0, hint, check);
+  last_block_pick(hist, nbits, st, level, 0);
 }
 
 // Segments of kSeg coordinates; a warp owns kWarpRun consecutive coordinates and reads them as
 // kRows rows of 128 (lane l holds coordinates 4l .. 4l+3 of each row), so every load is a
 // coalesced float4 and the ascending order of a warp's run is (row, lane, component).
+constexpr int kSegThreads = 256;
+constexpr int kSeg = 16384;
 constexpr int kSegWarps = kSegThreads / 32;
 constexpr int kWarpRun = kSeg / kSegWarps;   // 2048
 constexpr int kRows = kWarpRun / 128;        // 16
@@ -393,7 +537,7 @@ constexpr int kRows = kWarpRun / 128;        // 16
 template <bool VEC>
 __device__ __forceinline__ void load_row(const float* __restrict__ est, int64_t i0, int64_t s1, float (&v)[4]) {
   if (VEC && i0 + 4 <= s1) {
-    const float4 f = __ldcg(reinterpret_cast<const float4*>(est + i0));
+    const float4 f = __ldg(reinterpret_cast<const float4*>(est + i0));
     v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
   } else {
 #pragma unroll
@@ -406,16 +550,10 @@ __device__ __forceinline__ uint32_t count_key(uint32_t key, uint32_t tau) {
   return (key > tau ? 1u : 0u) | (key == tau ? (1u << 16) : 0u);
 }
 
-// The state whose threshold is valid: the exact re-run's when the first pass failed.
-__device__ __forceinline__ const SelectState* valid_state(const SelectState* st, const SelectState* st2) {
-  return (st2 && __ldcg(&st->fail)) ? st2 : st;
-}
-
 template <bool VEC>
 __global__ void __launch_bounds__(kSegThreads) k_count(const float* __restrict__ est, int64_t d,
-                                                       const SelectState* st0, const SelectState* st2,
-                                                       uint32_t* blk_gt, uint32_t* blk_eq) {
-  const SelectState* st = valid_state(st0, st2);
+                                                       const SelectState* st, uint32_t* blk_gt,
+                                                       uint32_t* blk_eq) {
   const uint32_t tau = __ldcg(&st->tau);
   const int64_t s0 = (int64_t)blockIdx.x * kSeg;
   const int64_t s1 = s0 + kSeg < d ? s0 + kSeg : d;
@@ -440,60 +578,13 @@ __global__ void __launch_bounds__(kSegThreads) k_count(const float* __restrict__
   }
 }
 
-__global__ void __launch_bounds__(kScanThreads) k_scan(const uint32_t* __restrict__ blk_gt,
-                                                       const uint32_t* __restrict__ blk_eq, int64_t nblk,
-                                                       const SelectState* st0, const SelectState* st2,
-                                                       uint32_t* blk_base, uint32_t* blk_eqx) {
-  const SelectState* st = valid_state(st0, st2);
-  const uint32_t need_eq = __ldcg(&st->need_eq);
-  uint32_t carry_gt = 0, carry_eq = 0;
-  for (int64_t c0 = 0; c0 < nblk; c0 += blockDim.x) {
-    const int64_t b = c0 + threadIdx.x;
-    const uint32_t g = b < nblk ? blk_gt[b] : 0u;
-    const uint32_t e = b < nblk ? blk_eq[b] : 0u;
-    uint32_t tg, te;
-    const uint32_t xg = block_excl_scan(g, &tg) + carry_gt;
-    const uint32_t xe = block_excl_scan(e, &te) + carry_eq;
-    if (b < nblk) {
-      blk_base[b] = xg + (xe < need_eq ? xe : need_eq);
-      blk_eqx[b] = xe;
-    }
-    carry_gt += tg;
-    carry_eq += te;
-  }
-}
-
-// Warp-inclusive scan of a packed count.
-__device__ __forceinline__ uint32_t warp_incl_scan(uint32_t x) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
-    if (lane >= o) x += y;
-  }
-  return x;
-}
-
-template <bool VEC>
-__device__ __forceinline__ void load_row_l1(const float* __restrict__ est, int64_t i0, int64_t s1, float (&v)[4]) {
-  if (VEC && i0 + 4 <= s1) {
-    const float4 f = __ldg(reinterpret_cast<const float4*>(est + i0));
-    v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
-  } else {
-#pragma unroll
-    for (int t = 0; t < 4; ++t) v[t] = (i0 + t < s1) ? est[i0 + t] : 0.f;
-  }
-}
-
 // Counts first (all rows in flight), then each row again from L1 to place its keys.
 template <bool VEC>
 __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__ est, int64_t d,
-                                                       const SelectState* st0, const SelectState* st2,
-                                                       const uint32_t* __restrict__ blk_base,
+                                                       const SelectState* st, const uint32_t* __restrict__ blk_base,
                                                        const uint32_t* __restrict__ blk_eqx,
                                                        int64_t* __restrict__ idx_out, int64_t k) {
   __shared__ uint32_t warp_tot[kSegWarps];
-  const SelectState* st = valid_state(st0, st2);
   const uint32_t tau = __ldcg(&st->tau), need_eq = __ldcg(&st->need_eq);
   const int64_t s0 = (int64_t)blockIdx.x * kSeg;
   const int64_t s1 = s0 + kSeg < d ? s0 + kSeg : d;
@@ -505,7 +596,7 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
   {
     float v[kRows][4];
 #pragma unroll
-    for (int j = 0; j < kRows; ++j) load_row_l1<VEC>(est, w0 + j * 128 + lane * 4, s1, v[j]);
+    for (int j = 0; j < kRows; ++j) load_row<VEC>(est, w0 + j * 128 + lane * 4, s1, v[j]);
 #pragma unroll
     for (int j = 0; j < kRows; ++j) {
 #pragma unroll
@@ -515,7 +606,7 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
     }
   }
   // warp totals -> each warp's prefix inside the segment
-  const uint32_t wsum = __shfl_sync(0xFFFFFFFFu, warp_incl_scan(cnt), 31);
+  const uint32_t wsum = __shfl_sync(kFull, warp_incl_scan(cnt), 31);
   if (lane == 0) warp_tot[warp] = wsum;
   __syncthreads();
   uint32_t wpre = 0;
@@ -527,7 +618,7 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
   for (int j = 0; j < kRows; ++j) {
     const int64_t i0 = w0 + j * 128 + lane * 4;
     float v[4];
-    load_row_l1<VEC>(est, i0, s1, v);
+    load_row<VEC>(est, i0, s1, v);
     uint32_t key[4];
     uint32_t c = 0;
 #pragma unroll
@@ -536,7 +627,7 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
       if (i0 + t < s1) c += count_key(key[t], tau);
     }
     const uint32_t incl = warp_incl_scan(c);
-    const uint32_t row_tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
+    const uint32_t row_tot = __shfl_sync(kFull, incl, 31);
     if (c) {
       const uint32_t before = run + incl - c;
       const uint32_t gt_before = before & 0xFFFFu, eq_before = before >> 16;
@@ -561,51 +652,40 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
   }
 }
 
-template <int R, bool PRUNE>
+// ---- launchers -----------------------------------------------------------------------------
+
+template <typename K>
+int persistent_grid(K kernel, int64_t work_items, int block) {
+  const int64_t need = (work_items + block - 1) / block;
+  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)kernel, block);
+  return (int)(need < 1 ? 1 : (need < cap ? need : cap));
+}
+
+template <int R>
 cudaError_t launch_query_r(const QueryParams& p, cudaStream_t s) {
-  auto kern = k_query<R, PRUNE>;
-  const int64_t need = ((p.d + 3) / 4 + kBlock - 1) / kBlock;
-  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)kern, kBlock);
-  const int grid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
-  kern<<<grid, kBlock, 0, s>>>(p);
+  auto kern = k_query<R>;
+  kern<<<persistent_grid(kern, (p.d + 3) / 4, kBlock), kBlock, 0, s>>>(p);
   return cudaGetLastError();
 }
 
 typedef cudaError_t (*QueryLauncher)(const QueryParams&, cudaStream_t);
 
-template <bool PRUNE, int... Rs>
+template <int... Rs>
 struct QueryTable {
-  static constexpr QueryLauncher table[sizeof...(Rs)] = {&launch_query_r<Rs, PRUNE>...};
+  static constexpr QueryLauncher table[sizeof...(Rs)] = {&launch_query_r<Rs>...};
 };
-template <bool PRUNE, int... Rs>
-constexpr QueryLauncher QueryTable<PRUNE, Rs...>::table[sizeof...(Rs)];
+template <int... Rs>
+constexpr QueryLauncher QueryTable<Rs...>::table[sizeof...(Rs)];
 
-cudaError_t launch_query(const QueryParams& p, bool prune, cudaStream_t s) {
-  using T = QueryTable<false, 1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
-  using TP = QueryTable<true, 1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
-  if (is_pow2(p.c) && p.r >= 1 && p.r <= GS_MAX_ROWS) return (prune ? TP::table : T::table)[p.r - 1](p, s);
-  const int64_t need = (p.d + kBlock - 1) / kBlock;
-  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)k_query_generic, kBlock);
-  const int grid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
-  k_query_generic<<<grid, kBlock, 0, s>>>(p);
+cudaError_t launch_query(const QueryParams& p, cudaStream_t s) {
+  using T = QueryTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
+  if (is_pow2(p.c) && p.r >= 1 && p.r <= GS_MAX_ROWS) return T::table[p.r - 1](p, s);
+  k_query_generic<<<persistent_grid(k_query_generic, p.d, kBlock), kBlock, 0, s>>>(p);
   return cudaGetLastError();
 }
 
-// The query and selection kernels over scratch laid out by the caller.  With `hint`
-// (requires hist of 6 * kBins and two states) the first pass prunes against the hint and
-// an exact re-run follows, gated on the first pass's fail flag; k_count, k_scan and k_write
-// then use whichever state is valid.
-cudaError_t run_query_select(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
-                             int64_t k, int64_t* idx_out, float* est, uint32_t* hist, SelectState* st,
-                             SelectState* st2, uint32_t* hint, uint32_t* blk_gt, uint32_t* blk_eq,
-                             uint32_t* blk_base, uint32_t* blk_eqx, cudaStream_t s) {
-  const bool vec = (reinterpret_cast<uintptr_t>(est) & 15u) == 0;
-  const bool prune = hint != nullptr && st2 != nullptr && is_pow2(c);
-  cudaError_t err = cudaMemsetAsync(hist, 0, (prune ? 6 : 3) * kBins * sizeof(uint32_t), s);
-  if (err != cudaSuccess) return err;
-  if ((err = cudaMemsetAsync(st, 0, sizeof(SelectState), s)) != cudaSuccess) return err;
-  if (prune && (err = cudaMemsetAsync(st2, 0, sizeof(SelectState), s)) != cudaSuccess) return err;
-
+QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
+                              int64_t k, float* est, uint32_t* hist, SelectState* st) {
   QueryParams qp;
   qp.T = merged;
   qp.est = est;
@@ -616,60 +696,83 @@ cudaError_t run_query_select(const float* merged, const HashCoeffs& h, int r, ui
   qp.r = r;
   qp.c = c;
   qp.cmask = c - 1;
-  qp.vec = vec ? 1 : 0;
-  qp.gate = nullptr;
-  qp.hint = hint;
+  qp.vec = (reinterpret_cast<uintptr_t>(est) & 15u) == 0 ? 1 : 0;
   qp.h = h;
-  if ((err = launch_query(qp, prune, s)) != cudaSuccess) return err;
+  return qp;
+}
 
-  const int64_t nq = (d + 3) / 4;
-  const int64_t need = (nq + kBlock - 1) / kBlock;
-  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)k_hist, kBlock);
-  const int hgrid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
-  k_hist<<<hgrid, kBlock, 0, s>>>(est, d, vec ? 1 : 0, st, hist + kBins, 9, 11, 1, nullptr, nullptr, 0);
-  k_hist<<<hgrid, kBlock, 0, s>>>(est, d, vec ? 1 : 0, st, hist + 2 * kBins, 0, 9, 2, nullptr,
-                                  prune ? hint : nullptr, 1);
-  if (prune) {  // exact re-run, a no-op unless the first pass failed
-    QueryParams q2 = qp;
-    q2.hist = hist + 3 * kBins;
-    q2.st = st2;
-    q2.gate = &st->fail;
-    q2.hint = nullptr;
-    if ((err = launch_query(q2, false, s)) != cudaSuccess) return err;
-    k_hist<<<hgrid, kBlock, 0, s>>>(est, d, vec ? 1 : 0, st2, hist + 4 * kBins, 9, 11, 1, &st->fail, nullptr, 0);
-    k_hist<<<hgrid, kBlock, 0, s>>>(est, d, vec ? 1 : 0, st2, hist + 5 * kBins, 0, 9, 2, &st->fail, hint, 0);
-  }
-  SelectState* s2 = prune ? st2 : nullptr;
+// Layout of the caller's workspace for the candidate pipeline.
+struct Workspace {
+  float* est;         // d
+  uint32_t* hist;     // 3 * kBins
+  SelectState* st;
+  uint2* cand;        // d (index, key) pairs: room for every coordinate
+  uint32_t* gt_bm;    // nbw words
+  uint32_t* eq_bm;    // nbw words
+  uint32_t* blk;      // 4 * nblk
+  int64_t nbw, nblk;
+};
 
-  const int64_t nblk = (d + kSeg - 1) / kSeg;
-  const int nb = (int)nblk;
-  if (vec) k_count<true><<<nb, kSegThreads, 0, s>>>(est, d, st, s2, blk_gt, blk_eq);
-  else k_count<false><<<nb, kSegThreads, 0, s>>>(est, d, st, s2, blk_gt, blk_eq);
-  k_scan<<<1, kScanThreads, 0, s>>>(blk_gt, blk_eq, nblk, st, s2, blk_base, blk_eqx);
-  if (vec) k_write<true><<<nb, kSegThreads, 0, s>>>(est, d, st, s2, blk_base, blk_eqx, idx_out, k);
-  else k_write<false><<<nb, kSegThreads, 0, s>>>(est, d, st, s2, blk_base, blk_eqx, idx_out, k);
-  return cudaGetLastError();
+Workspace carve(void* base, int64_t d) {
+  Workspace w;
+  char* p = static_cast<char*>(base);
+  w.nbw = (d + 31) / 32;
+  w.nblk = (w.nbw + kBmWords - 1) / kBmWords;
+  w.est = reinterpret_cast<float*>(p);
+  p += align256((size_t)d * sizeof(float));
+  w.hist = reinterpret_cast<uint32_t*>(p);
+  p += align256(3 * kBins * sizeof(uint32_t));
+  w.st = reinterpret_cast<SelectState*>(p);
+  p += align256(sizeof(SelectState));
+  w.cand = reinterpret_cast<uint2*>(p);
+  p += align256((size_t)d * sizeof(uint2));
+  w.gt_bm = reinterpret_cast<uint32_t*>(p);
+  p += align256((size_t)w.nbw * sizeof(uint32_t));
+  w.eq_bm = reinterpret_cast<uint32_t*>(p);
+  p += align256((size_t)w.nbw * sizeof(uint32_t));
+  w.blk = reinterpret_cast<uint32_t*>(p);
+  return w;
 }
 
 }  // namespace
 
 size_t query_topk_workspace_bytes(int64_t d, int64_t k) {
   (void)k;
-  const int64_t nblk = (d + kSeg - 1) / kSeg;
-  return align256((size_t)d * sizeof(float)) + align256(6 * kBins * sizeof(uint32_t)) +
-         2 * align256(sizeof(SelectState)) + align256((size_t)nblk * 4 * sizeof(uint32_t));
+  const int64_t nbw = (d + 31) / 32;
+  const int64_t nblk = (nbw + kBmWords - 1) / kBmWords;
+  return align256((size_t)d * sizeof(float)) + align256(3 * kBins * sizeof(uint32_t)) +
+         align256(sizeof(SelectState)) + align256((size_t)d * sizeof(uint2)) +
+         2 * align256((size_t)nbw * sizeof(uint32_t)) + align256((size_t)nblk * 4 * sizeof(uint32_t));
 }
 
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, uint32_t* hint, cudaStream_t s) {
+                              void* workspace, cudaStream_t s) {
   Workspace w = carve(workspace, d);
   float* est = est_out ? est_out : w.est;
-  // pruning only when est is internal: a caller asking for est gets every median exactly
-  uint32_t* h2 = est_out ? nullptr : hint;
-  SelectState* st2 = reinterpret_cast<SelectState*>(reinterpret_cast<char*>(w.st) + align256(sizeof(SelectState)));
-  return run_query_select(merged, h, r, c, d, k, idx_out, est, w.hist, w.st, st2, h2, w.blk_gt, w.blk_eq,
-                          w.blk_base, w.blk_eqx, s);
+  cudaError_t err = cudaMemsetAsync(w.hist, 0, 3 * kBins * sizeof(uint32_t), s);
+  if (err == cudaSuccess) err = cudaMemsetAsync(w.st, 0, sizeof(SelectState), s);
+  // the two bitmaps are adjacent: clear both at once
+  if (err == cudaSuccess)
+    err = cudaMemsetAsync(w.gt_bm, 0, (size_t)(reinterpret_cast<char*>(w.blk) - reinterpret_cast<char*>(w.gt_bm)), s);
+  if (err != cudaSuccess) return err;
+
+  const QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
+  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
+  k_cand<<<persistent_grid(k_cand, (d + 3) / 4 / kU, kBlock), kBlock, 0, s>>>(est, d, qp.vec, w.st, w.hist + kBins,
+                                                                                 w.cand, w.gt_bm);
+  const int small_grid = device_info().sms;
+  k_cand_hist3<<<small_grid, kBlock, 0, s>>>(w.cand, w.st, w.hist + 2 * kBins);
+  k_cand_mark<<<small_grid, kBlock, 0, s>>>(w.cand, w.st, w.gt_bm, w.eq_bm);
+  uint32_t* blk_gt = w.blk;
+  uint32_t* blk_eq = blk_gt + w.nblk;
+  uint32_t* blk_base = blk_eq + w.nblk;
+  uint32_t* blk_eqx = blk_base + w.nblk;
+  const int nb = (int)w.nblk;
+  k_bm_count<<<nb, kBmThreads, 0, s>>>(w.gt_bm, w.eq_bm, w.nbw, blk_gt, blk_eq);
+  k_scan<<<1, kScanThreads, 0, s>>>(blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx);
+  k_bm_write<<<nb, kBmThreads, 0, s>>>(w.gt_bm, w.eq_bm, w.nbw, w.st, blk_base, blk_eqx, idx_out, k);
+  return cudaGetLastError();
 }
 
 // ---- scratch without allocation ---------------------------------------------------------
@@ -718,15 +821,28 @@ cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, 
   char* p = static_cast<char*>(base);
   uint32_t* hist = reinterpret_cast<uint32_t*>(p);
   SelectState* st = reinterpret_cast<SelectState*>(p + kNoallocHistBytes);
-  const int64_t nblk = (d + kSeg - 1) / kSeg;
+  const int64_t nseg = (d + kSeg - 1) / kSeg;
   uint32_t* blk_gt = reinterpret_cast<uint32_t*>(p + kNoallocHistBytes + kNoallocStateBytes);
-  uint32_t* blk_eq = blk_gt + nblk;
-  uint32_t* blk_base = blk_eq + nblk;
-  uint32_t* blk_eqx = blk_base + nblk;
-  // the histograms and the state are cleared at the start of the sequence; the segment
-  // counters are fully overwritten
-  return run_query_select(merged, h, r, c, d, k, idx_out, est_out, hist, st, nullptr, nullptr, blk_gt, blk_eq,
-                          blk_base, blk_eqx, s);
+  uint32_t* blk_eq = blk_gt + nseg;
+  uint32_t* blk_base = blk_eq + nseg;
+  uint32_t* blk_eqx = blk_base + nseg;
+  // the histograms and the state must start at zero; the segment counters are overwritten
+  err = cudaMemsetAsync(hist, 0, kNoallocHistBytes, s);
+  if (err == cudaSuccess) err = cudaMemsetAsync(st, 0, sizeof(SelectState), s);
+  if (err != cudaSuccess) return err;
+
+  const QueryParams qp = make_query_params(merged, h, r, c, d, k, est_out, hist, st);
+  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
+  const int hgrid = persistent_grid(k_hist, (d + 3) / 4 / kU, kBlock);
+  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + kBins, 9, 11, 1);
+  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + 2 * kBins, 0, 9, 2);
+  const int nb = (int)nseg;
+  if (qp.vec) k_count<true><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_gt, blk_eq);
+  else k_count<false><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_gt, blk_eq);
+  k_scan<<<1, kScanThreads, 0, s>>>(blk_gt, blk_eq, nseg, st, blk_base, blk_eqx);
+  if (qp.vec) k_write<true><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_base, blk_eqx, idx_out, k);
+  else k_write<false><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_base, blk_eqx, idx_out, k);
+  return cudaGetLastError();
 }
 
 }  // namespace gs

@@ -316,10 +316,10 @@ def test_step_host_buffers(gs, H, kind):
 
 
 @pytest.mark.parametrize("r", [5, 4, 7])
-def test_pruned_query_matches_exact(gs, H, r):
-    """With est_out = NULL the query may skip rows against the previous call's threshold
-    hint; the selection must equal the unpruned query's on the same merged table and agree
-    with the oracle -- also when the threshold collapses below the hint (exact re-run)."""
+def test_internal_estimate_query_matches(gs, H, r):
+    """Steps whose estimate stays in the workspace (est_out = NULL) select exactly what a
+    query returning the estimate selects on the same merged table, and agree with the oracle,
+    also across a step where the state is cleared and the threshold collapses."""
     w = workloads.get_config("resnet18")
     P, d, c, k, seed = 4, 400_003, 1 << 13, 500, 91
     coeffs = oracle.derive_coefficients(r, seed)
@@ -338,10 +338,10 @@ def test_pruned_query_matches_exact(gs, H, r):
             es0 = [H.host(e) for e in run.es]
             gs.gs_step(run.sketch, run.us, run.es, [_dev(g) for g in grads], d, w.rho, k, run.idx, run.vals,
                        None, run.ws)
-            gs.gs_query_topk(run.sketch, d, k, idx_exact, run.est, ws_q)   # unpruned, same merged table
+            gs.gs_query_topk(run.sketch, d, k, idx_exact, run.est, ws_q)   # same merged table, est returned
             torch.cuda.synchronize()
             idx = H.host(run.idx)
-            assert np.array_equal(idx, H.host(idx_exact)), f"step {t}: pruned selection differs"
+            assert np.array_equal(idx, H.host(idx_exact)), f"step {t}: selections differ"
             H.check_selection_exact(idx, H.host(run.est), k)
             res = oracle.step(us0, es0, grads, w.rho, coeffs, c, k)
             band = oracle.cell_band(res.merged_abs, coeffs, np.arange(d))
