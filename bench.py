@@ -145,6 +145,29 @@ def k1_traffic_per_launch():
     return float(m_tr.group(1))
 
 
+# ---- ranks --------------------------------------------------------------------------------
+
+def dist_max(x: float, device=None) -> float:
+    """The maximum of x over all ranks (x itself without an initialised process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_workers(rank: int, P: int) -> list:
+    """Worker ids whose gradients rank `rank` draws: independent replicas per rank."""
+    return [rank * P + p for p in range(P)]
+
+
+def whole_job_rate(world: int, P: int, d: int, steps: int, max_seconds: float) -> float:
+    """Worker-coordinates of all ranks per second of the slowest rank."""
+    return world * P * d * steps / max_seconds
+
+
 # ---- our arm -----------------------------------------------------------------------------
 
 def gpu_uuid(dev) -> str:
@@ -188,12 +211,12 @@ def run_ours(args):
     host_pool, dev_pool = [], []
     for t in range(nsteps_pool):
         if host_gen:
-            gl = workloads.make_gradients(w, t, [rank * P + p for p in range(P)])
+            gl = workloads.make_gradients(w, t, replica_workers(rank, P))
             host_pool.append([torch.from_numpy(g).pin_memory() for g in gl])
             dev_pool.append([g.to(dev, non_blocking=True) for g in host_pool[-1]])
         else:
-            dev_pool.append([workloads.make_gradient_torch(w, t, rank * P + p, torch.empty(d, device=dev))
-                             for p in range(P)])
+            dev_pool.append([workloads.make_gradient_torch(w, t, q, torch.empty(d, device=dev))
+                             for q in replica_workers(rank, P)])
     if not host_gen and not args.no_e2e and not args.profile_steps:
         host_pool = [[g.cpu().pin_memory() for g in dev_pool[0]]]
     us = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
@@ -248,22 +271,19 @@ def run_ours(args):
         step(args.warmup + t, True)
     end.record(stream)
     torch.cuda.synchronize()
-    if sampler:
-        sampler.mark_end()
-    elapsed_ms = start.elapsed_time(end)
     if world > 1:
         import torch.distributed as dist
-        tt = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         dist.barrier()
-        elapsed_ms = float(tt.item())
+    if sampler:
+        sampler.mark_end()
+    elapsed_ms = dist_max(start.elapsed_time(end), dev)
     if sampler:
         clocks = sampler.stop()
 
     k1_ms = [a.elapsed_time(b) for a, b, _ in k1_events]
     k1_lanes = [n for _, _, n in k1_events]
     coords = world * P * d * args.steps
-    value = coords / (elapsed_ms / 1e3)
+    value = whole_job_rate(world, P, d, args.steps, elapsed_ms / 1e3)
 
     # roofline of the dominant kernel: fused accumulate + insert (20 algorithmic HBM bytes per
     # worker-coordinate: read g, u, e; write u, e)
@@ -313,10 +333,9 @@ def run_ours(args):
         e2e_s = time.perf_counter() - t0
         if world > 1:
             import torch.distributed as dist
-            tt = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e2e_s = float(tt.item())
-        e2e = {"value": coords / e2e_s, "unit": UNIT, "h2d_bytes_per_step": P * d * 4,
+            dist.barrier()
+        e2e_s = dist_max(e2e_s, dev)
+        e2e = {"value": whole_job_rate(world, P, d, args.steps, e2e_s), "unit": UNIT, "h2d_bytes_per_step": P * d * 4,
                "d2h_bytes_per_step": k * (8 + 4), "ms_per_step": round(e2e_s * 1e3 / args.steps, 4),
                "call": "gs_step_host"}
 
