@@ -148,6 +148,22 @@ gs_status gs_query_topk(const gs_sketch* sketch, int64_t d, int64_t k, int64_t* 
                         float* est_out, void* workspace, size_t workspace_bytes,
                         gs_stream stream);
 
+/* Device workspace bytes gs_query_heavymix needs. */
+gs_status gs_query_heavymix_workspace_size(int64_t d, int64_t k, size_t* bytes);
+
+/* HEAVYMIX selection from the merged table, as Alg. 2 prints it.  With est_i the median query
+ * as in gs_query_topk and l2sq = the median over rows j of sum_b T[j][b]^2 (the sketch's
+ * estimate of ||g||_2^2), H = {i : est_i^2 >= l2sq / k} and NH its complement (Alg. 2 step 2).
+ * If |H| >= k the k coordinates of H with largest |est| are selected (ties to the smaller
+ * index); otherwise all of H and l = k - |H| coordinates of NH drawn uniformly at random
+ * (Alg. 2 step 3): those with the smallest xi_i = (i-th splitmix64 output of fill_seed) >> 33,
+ * i counted from 0, ties to the smaller index.  idx_out (int64[k]) is ascending; est_out
+ * (fp32[d]) and l2sq_out (one device double) may be NULL.  workspace must hold
+ * gs_query_heavymix_workspace_size(d, k) bytes, 256-byte aligned. */
+gs_status gs_query_heavymix(const gs_sketch* sketch, int64_t d, int64_t k, uint64_t fill_seed,
+                            int64_t* idx_out, float* est_out, double* l2sq_out, void* workspace,
+                            size_t workspace_bytes, gs_stream stream);
+
 /* Largest d that gs_query_topk_noalloc accepts. */
 #define GS_NOALLOC_MAX_DIM (1LL << 30)
 
@@ -180,6 +196,22 @@ gs_status gs_gather_and_zero(float* const* momentum, float* const* error, int32_
                              int64_t d, const int64_t* idx, int64_t k, float* vals_out,
                              gs_stream stream);
 
+/* ---- step 7: weight update ------------------------------------------------------- */
+
+/* w[idx[t]] <- fl(w[idx[t]] - fl(lr * vals[t])) for t < k: Alg. 1 step 26,
+ * w_{t+1} = w_t - eta * G~_t, with G~_t the gathered values at the selected indices and zero
+ * elsewhere (the values are sums over workers, so lr absorbs any averaging).  All workers hold
+ * the same weights, so one vector is updated.  idx holds distinct indices; indices outside
+ * [0, d) are skipped. */
+gs_status gs_apply_update(float* weights, int64_t d, const int64_t* idx, const float* vals,
+                          int64_t k, float lr, gs_stream stream);
+
+/* gs_gather_and_zero and, when weights is not NULL, gs_apply_update with the gathered values,
+ * in one kernel. */
+gs_status gs_gather_zero_update(float* const* momentum, float* const* error, int32_t P,
+                                int64_t d, const int64_t* idx, int64_t k, float* vals_out,
+                                float* weights, float lr, gs_stream stream);
+
 /* ---- whole step ------------------------------------------------------------------ */
 
 /* Device workspace bytes gs_step needs (query workspace plus the step's own buffers). */
@@ -194,6 +226,13 @@ gs_status gs_step(gs_sketch* sketch, float* const* momentum, float* const* error
                   const float* const* grad, int64_t d, float rho, int64_t k,
                   int64_t* idx_out, float* vals_out, float* est_out, void* workspace,
                   size_t workspace_bytes, gs_stream stream);
+
+/* gs_step followed by the weight update of Alg. 1 step 26 (fused into the gather):
+ * one training step of gs-SGD's compression and update for the simulated workers. */
+gs_status gs_train_step(gs_sketch* sketch, float* weights, float lr, float* const* momentum,
+                        float* const* error, const float* const* grad, int64_t d, float rho,
+                        int64_t k, int64_t* idx_out, float* vals_out, float* est_out,
+                        void* workspace, size_t workspace_bytes, gs_stream stream);
 
 /* gs_step with the gradients in HOST memory and the results returned to HOST memory, one
  * synchronous call per step.  Where the device can address grad_host[p] in place (memory

@@ -32,6 +32,7 @@ from .countsketch import (  # noqa: F401
     bucket_exact,
     sign_exact,
     hash_rows,
+    splitmix64_at,
 )
 from .gssgd import (  # noqa: F401
     accumulate,
@@ -41,7 +42,10 @@ from .gssgd import (  # noqa: F401
     query,
     cell_band,
     topk,
+    heavymix,
+    heavymix_select,
     gather_and_zero,
+    apply_update,
     step,
     StepResult,
 )

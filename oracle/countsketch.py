@@ -43,6 +43,18 @@ def splitmix64(seed: int):
         yield z ^ (z >> 31)
 
 
+def splitmix64_at(seed: int, idx) -> np.ndarray:
+    """The outputs number idx (0-based) of the splitmix64 stream seeded with ``seed``, as
+    uint64: the state after idx + 1 golden-ratio increments, mixed (counter-based form of the
+    same published generator)."""
+    with np.errstate(over="ignore"):
+        i = np.asarray(idx, dtype=np.uint64)
+        z = np.uint64(seed & _MASK64) + (i + np.uint64(1)) * np.uint64(0x9E3779B97F4A7C15)
+        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)
+        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
+        return z ^ (z >> np.uint64(31))
+
+
 def derive_coefficients(r: int, seed: int):
     """Coefficients (a, b, a2, b2), each a list of r Python ints, for rows 0..r-1.
 

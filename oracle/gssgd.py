@@ -17,6 +17,7 @@ Alg. 2 (HEAVYMIX) of the paper:
                   (Alg. 2 steps 2-3 read as a deterministic top-k, see the design notes)
   6. second round the exact values v_t = sum_p e_p[I_t] of the selected coordinates
                   (Alg. 2 step 4), after which u_p and e_p are zeroed at I_t.
+  7. update       w <- w - lr * G~, G~ = v at I and 0 elsewhere (Alg. 1 step 26)
 
 Sketch cells, merge, median and gathered values are computed in fp64; alongside each table
 the oracle keeps the table of absolute contributions (sum of |s*x| per cell), which sets
@@ -29,7 +30,7 @@ import dataclasses
 
 import numpy as np
 
-from .countsketch import hash_rows
+from .countsketch import hash_rows, splitmix64_at
 
 
 # ---- 1. accumulate ---------------------------------------------------------------------
@@ -149,6 +150,37 @@ def topk(est: np.ndarray, k: int) -> np.ndarray:
     return np.sort(order[:k]).astype(np.int64)
 
 
+# ---- 5'. HEAVYMIX ----------------------------------------------------------------------
+
+def heavymix_select(est: np.ndarray, l2sq: float, k: int, fill_seed: int) -> np.ndarray:
+    """Alg. 2 steps 2-3 from given estimates and ||g||^2 estimate (indices ascending):
+    H = {i : est_i^2 >= l2sq / k}, est_i taken at fp32 precision and squared exactly; if
+    |H| >= k the k members of H with largest |est| (ties to the smaller index), else H plus the
+    l = k - |H| members of NH with the smallest xi_i = splitmix64_at(fill_seed, i) >> 33,
+    ties to the smaller index (a uniformly random l-subset of NH)."""
+    est = np.asarray(est, dtype=np.float64)
+    est32 = est.astype(np.float32).astype(np.float64)
+    in_h = est32 * est32 >= l2sq / k
+    nh = int(in_h.sum())
+    if nh >= k:
+        return topk(np.where(in_h, est, 0.0), k)
+    NH = np.nonzero(~in_h)[0]
+    xi = (splitmix64_at(fill_seed, NH) >> np.uint64(33)).astype(np.int64)
+    fill = NH[np.lexsort((NH, xi))[: k - nh]]
+    return np.sort(np.concatenate([np.nonzero(in_h)[0], fill])).astype(np.int64)
+
+
+def heavymix(T: np.ndarray, coeffs, d: int, k: int, fill_seed: int, hashes=None):
+    """Alg. 2 steps 1-3 as printed (returns idx ascending, est, l2sq): est is the median query
+    (step 1); l2sq, the median over rows j of sum_b T[j][b]^2, estimates ||g||_2^2; the
+    selection is ``heavymix_select`` (steps 2-3)."""
+    est = query(T, coeffs, d, hashes)
+    rows = np.sort(np.sum(np.asarray(T, dtype=np.float64) ** 2, axis=1))
+    r = rows.size
+    l2sq = rows[r // 2] if r % 2 == 1 else 0.5 * (rows[r // 2 - 1] + rows[r // 2])
+    return heavymix_select(est, l2sq, k, fill_seed), est, l2sq
+
+
 # ---- 6. second round: gather exact values and zero the accumulators ---------------------
 
 def gather_and_zero(us, es, idx):
@@ -169,6 +201,21 @@ def gather_and_zero(us, es, idx):
         us_out.append(u2)
         es_out.append(e2)
     return vals, us_out, es_out
+
+
+# ---- 7. weight update ------------------------------------------------------------------
+
+def apply_update(w: np.ndarray, idx, vals, lr: float) -> np.ndarray:
+    """Alg. 1 step 26, w <- w - lr * G~ with G~ = vals at idx and 0 elsewhere, in fp32
+    semantics: w'[i] = fl(w[i] - fl(lr * v)) with lr taken as the nearest fp32 value.  The
+    input is not modified; idx must hold distinct indices."""
+    w2 = np.array(w, dtype=np.float32, copy=True)
+    idx = np.asarray(idx, dtype=np.int64)
+    lr64 = np.float64(np.float32(lr))
+    v64 = np.asarray(vals, dtype=np.float32).astype(np.float64)
+    step = (lr64 * v64).astype(np.float32).astype(np.float64)
+    w2[idx] = (w2[idx].astype(np.float64) - step).astype(np.float32)
+    return w2
 
 
 # ---- one full step ---------------------------------------------------------------------

@@ -47,7 +47,12 @@ SIGNATURES = {
     "gs_query_topk_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_query_topk": [_vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp],
     "gs_query_topk_noalloc": [_vp, _i64, _i64, _vp, _vp, _vp],
+    "gs_query_heavymix_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
+    "gs_query_heavymix": [_vp, _i64, _i64, _u64, _vp, _vp, _vp, _vp, _sz, _vp],
     "gs_gather_and_zero": [_PP, _PP, _i32, _i64, _vp, _i64, _vp, _vp],
+    "gs_apply_update": [_vp, _i64, _vp, _vp, _i64, _f32, _vp],
+    "gs_gather_zero_update": [_PP, _PP, _i32, _i64, _vp, _i64, _vp, _vp, _f32, _vp],
+    "gs_train_step": [_vp, _vp, _f32, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
     "gs_step_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_step": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
     "gs_step_host": [_vp, _PP, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _sz, _vp],
@@ -177,6 +182,21 @@ def gs_query_topk(sketch: int, d: int, k: int, idx_out, est_out, workspace, work
                                         workspace_bytes, _stream(stream)), "gs_query_topk")
 
 
+def gs_query_heavymix_workspace_size(d: int, k: int) -> int:
+    out = _sz()
+    _check(load_library().gs_query_heavymix_workspace_size(d, k, ctypes.byref(out)),
+           "gs_query_heavymix_workspace_size")
+    return out.value
+
+
+def gs_query_heavymix(sketch: int, d: int, k: int, fill_seed: int, idx_out, est_out, l2sq_out, workspace,
+                      workspace_bytes=None, stream=None) -> None:
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(load_library().gs_query_heavymix(sketch, d, k, fill_seed, _ptr(idx_out), _ptr(est_out), _ptr(l2sq_out),
+                                            _ptr(workspace), workspace_bytes, _stream(stream)), "gs_query_heavymix")
+
+
 def gs_query_topk_noalloc(sketch: int, d: int, k: int, idx_out, est_out, stream=None) -> None:
     """gs_query_topk without a caller workspace: the library's fixed device scratch is used
     (for hosts that cannot allocate device memory; est_out is required)."""
@@ -188,6 +208,28 @@ def gs_gather_and_zero(momentum, error, d: int, idx, k: int, vals_out, stream=No
     P = len(momentum)
     _check(load_library().gs_gather_and_zero(_ptr_array(momentum), _ptr_array(error), P, d, _ptr(idx), k,
                                              _ptr(vals_out), _stream(stream)), "gs_gather_and_zero")
+
+
+def gs_apply_update(weights, d: int, idx, vals, k: int, lr: float, stream=None) -> None:
+    _check(load_library().gs_apply_update(_ptr(weights), d, _ptr(idx), _ptr(vals), k, lr, _stream(stream)),
+           "gs_apply_update")
+
+
+def gs_gather_zero_update(momentum, error, d: int, idx, k: int, vals_out, weights, lr: float,
+                          stream=None) -> None:
+    P = len(momentum)
+    _check(load_library().gs_gather_zero_update(_ptr_array(momentum), _ptr_array(error), P, d, _ptr(idx), k,
+                                                _ptr(vals_out), _ptr(weights), lr, _stream(stream)),
+           "gs_gather_zero_update")
+
+
+def gs_train_step(sketch: int, weights, lr: float, momentum, error, grad, d: int, rho: float, k: int,
+                  idx_out, vals_out, est_out, workspace, workspace_bytes=None, stream=None) -> None:
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(load_library().gs_train_step(sketch, _ptr(weights), lr, _ptr_array(momentum), _ptr_array(error),
+                                        _ptr_array(grad), d, rho, k, _ptr(idx_out), _ptr(vals_out), _ptr(est_out),
+                                        _ptr(workspace), workspace_bytes, _stream(stream)), "gs_train_step")
 
 
 def gs_step_workspace_size(d: int, k: int) -> int:

@@ -164,7 +164,7 @@ gs_status accumulate_insert_impl(gs_sketch* sk, int32_t first, int32_t n, float*
 
 gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float* const* g,
                     int64_t d, float rho, int64_t k, int64_t* idx, float* vals, float* est,
-                    void* ws, cudaStream_t s) {
+                    void* ws, cudaStream_t s, float* weights = nullptr, float lr = 0.f) {
   const size_t bytes = (size_t)sk->groups * sk->r * sk->c * sk->W * sizeof(float) +
                        (size_t)sk->r * sk->c * sizeof(float);
   cudaError_t err = cudaMemsetAsync(sk->tables, 0, bytes, s);
@@ -188,6 +188,8 @@ gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float
   }
   gp.idx = idx;
   gp.vals = vals;
+  gp.w = weights;
+  gp.lr = lr;
   gp.k = k;
   gp.d = d;
   gp.P = sk->workers;
@@ -428,6 +430,32 @@ gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_
   return GS_OK;
 }
 
+gs_status gs_query_heavymix_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = gs::heavymix_workspace_bytes(d, k);
+  return GS_OK;
+}
+
+gs_status gs_query_heavymix(const gs_sketch* sk, int64_t d, int64_t k, uint64_t fill_seed, int64_t* idx_out,
+                            float* est_out, double* l2sq_out, void* workspace, size_t workspace_bytes,
+                            gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  if (est_out) GS_TRY(check_vec(est_out, "est_out"));
+  if (l2sq_out && !aligned(l2sq_out, 8)) return fail(GS_ERR_INVALID_ARG, "l2sq_out is not 8-byte aligned");
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < gs::heavymix_workspace_bytes(d, k))
+    return fail(GS_ERR_INVALID_ARG, "workspace too small: need " + std::to_string(gs::heavymix_workspace_bytes(d, k)));
+  cudaError_t e = gs::launch_query_heavymix(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, fill_seed, idx_out,
+                                            est_out, l2sq_out, workspace, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "HEAVYMIX launch");
+  return GS_OK;
+}
+
 gs_status gs_query_topk_noalloc(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_out, float* est_out,
                                 gs_stream stream) {
   GS_TRY(check_sketch(sk));
@@ -463,6 +491,8 @@ gs_status gs_gather_and_zero(float* const* momentum, float* const* error, int32_
   }
   gp.idx = idx;
   gp.vals = vals_out;
+  gp.w = nullptr;
+  gp.lr = 0.f;
   gp.k = k;
   gp.d = d;
   gp.P = P;
@@ -470,6 +500,47 @@ gs_status gs_gather_and_zero(float* const* momentum, float* const* error, int32_
   if (e != cudaSuccess) return cuda_fail(e, "gather launch");
   return GS_OK;
   GS_GUARD_END
+}
+
+gs_status gs_gather_zero_update(float* const* momentum, float* const* error, int32_t P, int64_t d, const int64_t* idx,
+                                int64_t k, float* vals_out, float* weights, float lr, gs_stream stream) {
+  GS_GUARD_BEGIN
+  if (P < 1 || P > GS_MAX_WORKERS) return fail(GS_ERR_INVALID_ARG, "P must lie in [1, 64]");
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!idx || !aligned(idx, 8)) return fail(GS_ERR_INVALID_ARG, "idx is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals_out, "vals_out"));
+  if (weights) GS_TRY(check_vec(weights, "weights"));
+  GS_TRY(check_worker_arrays(P, momentum, error, nullptr));
+  gs::GatherParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  for (int p = 0; p < P; ++p) {
+    gp.u[p] = momentum[p];
+    gp.e[p] = error[p];
+  }
+  gp.idx = idx;
+  gp.vals = vals_out;
+  gp.w = weights;
+  gp.lr = lr;
+  gp.k = k;
+  gp.d = d;
+  gp.P = P;
+  cudaError_t e = gs::launch_gather_and_zero(gp, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "gather launch");
+  return GS_OK;
+  GS_GUARD_END
+}
+
+gs_status gs_apply_update(float* weights, int64_t d, const int64_t* idx, const float* vals, int64_t k, float lr,
+                          gs_stream stream) {
+  GS_TRY(check_vec(weights, "weights"));
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!idx || !aligned(idx, 8)) return fail(GS_ERR_INVALID_ARG, "idx is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals, "vals"));
+  cudaError_t e = gs::launch_apply_update(weights, d, idx, vals, k, lr, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "update launch");
+  return GS_OK;
 }
 
 gs_status gs_step_workspace_size(int64_t d, int64_t k, size_t* bytes) {
@@ -495,6 +566,26 @@ gs_status gs_step(gs_sketch* sk, float* const* momentum, float* const* error, co
   if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
   if (workspace_bytes < gs::query_topk_workspace_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small");
   return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, est_out, workspace, as_stream(stream));
+  GS_GUARD_END
+}
+
+gs_status gs_train_step(gs_sketch* sk, float* weights, float lr, float* const* momentum, float* const* error,
+                        const float* const* grad, int64_t d, float rho, int64_t k, int64_t* idx_out, float* vals_out,
+                        float* est_out, void* workspace, size_t workspace_bytes, gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  GS_TRY(check_vec(weights, "weights"));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad));
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals_out, "vals_out"));
+  if (est_out) GS_TRY(check_vec(est_out, "est_out"));
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < gs::query_topk_workspace_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small");
+  return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, est_out, workspace, as_stream(stream),
+                   weights, lr);
   GS_GUARD_END
 }
 

@@ -96,6 +96,8 @@ struct GatherParams {
   float* e[GS_MAX_WORKERS];
   const int64_t* idx;
   float* vals;
+  float* w;          // weights to update with the gathered values (nullable)
+  float lr;
   int64_t k, d;
   int32_t P;
 };
@@ -117,11 +119,20 @@ cudaError_t launch_hash_eval(const HashCoeffs& h, int r, uint32_t c, const int64
                              int64_t n, int32_t* bucket_out, int8_t* sign_out, cudaStream_t s);
 cudaError_t launch_merge(const MergeParams& p, int W, cudaStream_t s);
 cudaError_t launch_gather_and_zero(const GatherParams& p, cudaStream_t s);
+cudaError_t launch_apply_update(float* w, int64_t d, const int64_t* idx, const float* vals, int64_t k, float lr,
+                                cudaStream_t s);
 
 size_t query_topk_workspace_bytes(int64_t d, int64_t k);
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
                               void* workspace, cudaStream_t s);
+// HEAVYMIX selection (Alg. 2 as printed) from the merged table; l2sq_out (device double,
+// nullable) receives the sketch's estimate of ||g||^2.
+size_t heavymix_workspace_bytes(int64_t d, int64_t k);
+cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
+                                  int64_t k, uint64_t fill_seed, int64_t* idx_out, float* est_out, double* l2sq_out,
+                                  void* workspace, cudaStream_t s);
+
 // Same pipeline with its scratch in a fixed device array (no allocation); est_out required,
 // d <= GS_NOALLOC_MAX_DIM.  The first call on a device looks up the array's address.
 cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, int r, uint32_t c,

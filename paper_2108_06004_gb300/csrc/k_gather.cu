@@ -1,4 +1,6 @@
-// Step 6: the second round of Alg. 2 -- the exact values of the selected coordinates.
+// Step 6: the second round of Alg. 2 -- the exact values of the selected coordinates --
+// and step 7, the weight update of Alg. 1 (w <- w - lr * G~, G~ = the gathered values at the
+// selected indices and zero elsewhere), which the gather can apply on the fly.
 //
 // On a cluster the workers exchange their accumulated values at the k selected indices;
 // here every worker's error vector is on the device, so one thread per selected index
@@ -23,6 +25,7 @@ __global__ void __launch_bounds__(kBlock) k_gather_and_zero(const __grid_constan
     float v = 0.f;
     for (int p = 0; p < prm.P; ++p) v = __fadd_rn(v, prm.e[p][i]);
     prm.vals[t] = v;
+    if (prm.w) prm.w[i] = __fsub_rn(prm.w[i], __fmul_rn(prm.lr, v));
     for (int p = 0; p < prm.P; ++p) {
       prm.u[p][i] = 0.f;
       prm.e[p][i] = 0.f;
@@ -30,7 +33,27 @@ __global__ void __launch_bounds__(kBlock) k_gather_and_zero(const __grid_constan
   }
 }
 
+// w[idx[t]] <- fl(w[idx[t]] - fl(lr * vals[t])); indices outside [0, d) are skipped.
+__global__ void __launch_bounds__(kBlock) k_apply_update(float* __restrict__ w, int64_t d,
+                                                         const int64_t* __restrict__ idx,
+                                                         const float* __restrict__ vals, int64_t k, float lr) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < k; t += stride) {
+    const int64_t i = idx[t];
+    if (i >= 0 && i < d) w[i] = __fsub_rn(w[i], __fmul_rn(lr, vals[t]));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_apply_update(float* w, int64_t d, const int64_t* idx, const float* vals, int64_t k, float lr,
+                                cudaStream_t s) {
+  const int64_t need = (k + kBlock - 1) / kBlock;
+  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)k_apply_update, kBlock);
+  const int grid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
+  k_apply_update<<<grid, kBlock, 0, s>>>(w, d, idx, vals, k, lr);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_gather_and_zero(const GatherParams& p, cudaStream_t s) {
   const int64_t need = (p.k + kBlock - 1) / kBlock;

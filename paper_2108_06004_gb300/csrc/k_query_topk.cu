@@ -1,8 +1,9 @@
 // Steps 4 and 5: median-of-r query of the merged sketch and top-k selection
 // (Alg. 2 steps 1-3, read as a deterministic top-k by |est| with ties to the smaller index).
 //
-// The selection is a radix select on key = bits of |est| (for non-negative floats the bit
-// pattern orders like the value) in three levels: bits 30..20, 19..9 and 8..0.  Each
+// The selection is a radix select on a 32-bit key in three levels: bits 31..21, 20..10 and
+// 9..0.  For the top-k by |est| the key is the bit pattern of |est| (for non-negative floats
+// it orders like the value); HEAVYMIX selects on a composite key (see k_heavy_keys).  Each
 // histogram kernel ends with a pick: the last CTA to finish (found with a counter after a
 // memory fence, so no CTA waits for another) finds the bin that holds the k-th largest key
 // and how many keys of that bin are still to be taken.  After three levels the k-th largest
@@ -30,6 +31,9 @@ namespace gs {
 namespace {
 
 constexpr int kBins = 2048;
+constexpr int kL1Shift = 21;  // level 1: key bits 31..21 (11 bits)
+constexpr int kL2Shift = 10;  // level 2: key bits 20..10 (11 bits)
+constexpr int kL3Bits = 10;   // level 3: key bits 9..0
 constexpr int kScanThreads = 1024;
 constexpr uint32_t kNone = 0xFFFFFFFFu;
 constexpr uint32_t kFull = 0xFFFFFFFFu;
@@ -176,6 +180,7 @@ struct QueryParams {
   int32_t r;
   uint32_t c, cmask;
   int32_t vec;        // est 16-byte aligned
+  int32_t hist_on;    // build the level-1 histogram of |est| keys and pick
   HashCoeffs h;
 };
 
@@ -226,11 +231,15 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
       for (int t = 0; t < 4; ++t) m[t] = median_of<R>(v[t]);
       store_est(prm, i0, tmax, m);
     }
+    if (prm.hist_on) {
 #pragma unroll
-    for (int t = 0; t < 4; ++t) hist_add(sh, t < tmax ? (key_of(m[t]) >> 20) : kNone);
+      for (int t = 0; t < 4; ++t) hist_add(sh, t < tmax ? (key_of(m[t]) >> kL1Shift) : kNone);
+    }
   }
-  hist_flush(sh, prm.hist, kBins);
-  last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
+  if (prm.hist_on) {
+    hist_flush(sh, prm.hist, kBins);
+    last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
+  }
 }
 
 // General path: any r <= 16 and any c (bucket by 64-bit remainder).
@@ -264,12 +273,14 @@ __global__ void __launch_bounds__(kBlock) k_query_generic(const __grid_constant_
       }
       const float m = (r & 1) ? v[r / 2] : 0.5f * (v[r / 2 - 1] + v[r / 2]);
       prm.est[i] = m;
-      bin = key_of(m) >> 20;
+      bin = key_of(m) >> kL1Shift;
     }
-    hist_add(sh, bin);
+    if (prm.hist_on) hist_add(sh, bin);
   }
-  hist_flush(sh, prm.hist, kBins);
-  last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
+  if (prm.hist_on) {
+    hist_flush(sh, prm.hist, kBins);
+    last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
+  }
 }
 
 // Four float4 of est per thread in flight (kU strides of the grid-stride loop).
@@ -300,7 +311,8 @@ __device__ __forceinline__ void load_quads(const float* __restrict__ est, int64_
 // certain: their bit goes into gt_bm.  Keys inside the bin are appended to `cand` (index, key)
 // and feed the level-2 histogram; the level-2 pick follows.  A warp reserves room for all
 // candidates of its kU x 4 slots with a single atomic on the shared counter.
-__global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ est, int64_t d, int vec,
+// `src` holds the keys as 32-bit words: the bits of est (kmask drops the sign) or a key array.
+__global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ src, int64_t d, int vec, uint32_t kmask,
                                                  SelectState* st, uint32_t* hist2, uint2* __restrict__ cand,
                                                  uint32_t* gt_bm) {
   __shared__ uint32_t sh[kBins];
@@ -314,7 +326,7 @@ __global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ est, 
   for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += kU * stride) {
     float v[kU][4];
     int tm[kU];
-    load_quads(est, d, vec, q0, stride, v, tm);
+    load_quads(src, d, vec, q0, stride, v, tm);
     uint32_t keys[kU][4];
     uint32_t slot_mask[kU][4];
     uint32_t total = 0;
@@ -323,9 +335,9 @@ __global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ est, 
       const int64_t i0 = (q0 + u * stride + lane) * 4;
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
-        const uint32_t key = key_of(v[u][t]);
+        const uint32_t key = __float_as_uint(v[u][t]) & kmask;
         const bool valid = t < tm[u];
-        const uint32_t bin1 = key >> 20;
+        const uint32_t bin1 = key >> kL1Shift;
         const int64_t i = i0 + t;
         if (valid && bin1 > b1) atomicOr(&gt_bm[i >> 5], 1u << (i & 31));
         keys[u][t] = key;
@@ -346,7 +358,7 @@ __global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ est, 
         if (m) {
           const bool in = (m >> lane) & 1u;
           if (in) cand[base + __popc(m & lower)] = make_uint2((uint32_t)(i0 + t), keys[u][t]);
-          hist_add(sh, in ? ((keys[u][t] >> 9) & (kBins - 1)) : kNone);
+          hist_add(sh, in ? ((keys[u][t] >> kL2Shift) & (kBins - 1)) : kNone);
           base += __popc(m);
         }
       }
@@ -359,8 +371,9 @@ __global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ est, 
 // Level-3 histogram of the candidates that match the 22-bit prefix; the last pick gives tau.
 __global__ void __launch_bounds__(kBlock) k_cand_hist3(const uint2* __restrict__ cand, SelectState* st,
                                                        uint32_t* hist3) {
-  __shared__ uint32_t sh[512];
-  for (int b = threadIdx.x; b < 512; b += blockDim.x) sh[b] = 0;
+  constexpr int kN3 = 1 << kL3Bits;
+  __shared__ uint32_t sh[kN3];
+  for (int b = threadIdx.x; b < kN3; b += blockDim.x) sh[b] = 0;
   __syncthreads();
   const uint32_t n = __ldcg(&st->ncand);
   const uint32_t p22 = __ldcg(&st->prefix);
@@ -371,12 +384,12 @@ __global__ void __launch_bounds__(kBlock) k_cand_hist3(const uint2* __restrict__
     uint32_t bin = kNone;
     if (t < n) {
       const uint32_t key = cand[t].y;
-      if ((key >> 9) == p22) bin = key & 511u;
+      if ((key >> kL2Shift) == p22) bin = key & (uint32_t)(kN3 - 1);
     }
     if (__any_sync(kFull, bin != kNone)) hist_add(sh, bin);
   }
-  hist_flush(sh, hist3, 512);
-  last_block_pick(hist3, 9, st, 2, 0);
+  hist_flush(sh, hist3, kN3);
+  last_block_pick(hist3, kL3Bits, st, 2, 0);
 }
 
 // Candidates above tau into gt_bm, candidates equal to tau into eq_bm.
@@ -652,6 +665,93 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
   }
 }
 
+// ---- HEAVYMIX (Alg. 2 as printed) ----------------------------------------------------------
+
+// Sum of squares of each row of the merged table in fp64; blockIdx.y is the row.
+__global__ void __launch_bounds__(kBlock) k_row_sumsq(const float* __restrict__ T, uint32_t c, double* sumsq) {
+  __shared__ double warp_acc[kBlock / 32];
+  const int j = blockIdx.y;
+  const float* row = T + (size_t)j * c;
+  double acc = 0.0;
+  for (uint32_t b = blockIdx.x * blockDim.x + threadIdx.x; b < c; b += gridDim.x * blockDim.x) {
+    const double v = (double)row[b];
+    acc += v * v;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(kFull, acc, o);
+  if ((threadIdx.x & 31) == 0) warp_acc[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    double v = threadIdx.x < kBlock / 32 ? warp_acc[threadIdx.x] : 0.0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(kFull, v, o);
+    if (threadIdx.x == 0) atomicAdd(&sumsq[j], v);
+  }
+}
+
+// l2sq = median over rows of the row sums of squares (the sketch's estimate of ||g||^2);
+// theta = l2sq / k, the threshold of H.
+__global__ void k_heavy_theta(const double* __restrict__ sumsq, int r, int64_t k, double* theta,
+                              double* l2sq_out) {
+  if (blockIdx.x != 0 || threadIdx.x != 0) return;
+  double v[GS_MAX_ROWS];
+  for (int j = 0; j < r; ++j) v[j] = __ldcg(&sumsq[j]);
+  for (int a = 1; a < r; ++a) {
+    const double t = v[a];
+    int b = a - 1;
+    while (b >= 0 && v[b] > t) {
+      v[b + 1] = v[b];
+      --b;
+    }
+    v[b + 1] = t;
+  }
+  const double m = (r & 1) ? v[r / 2] : 0.5 * (v[r / 2 - 1] + v[r / 2]);
+  theta[0] = m / (double)k;
+  if (l2sq_out) l2sq_out[0] = m;
+}
+
+// The i-th output (i = 0, 1, ...) of the splitmix64 stream seeded with `seed`: the state after
+// i + 1 increments of the golden-ratio constant, mixed (Steele, Lea and Flood, 2014).
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t i) {
+  uint64_t z = seed + (i + 1) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Composite key of HEAVYMIX.  Members of H = {i : est_i^2 >= theta} get 0x80000000 | bits(|est_i|):
+// all of H ranks above all of NH, and inside H by |est|.  Members of NH get 0x7FFFFFFF - xi_i,
+// xi_i = the top 31 bits of splitmix64_at(fill_seed, i): the largest NH keys are the NH
+// coordinates with the smallest xi, a uniformly random subset (rand_l(NH)).  The top-k of these
+// keys (ties to the smaller index) is H plus k - |H| random coordinates of NH when |H| < k, and
+// the k largest |est| of H otherwise.  Ends with the level-1 histogram and pick.
+__global__ void __launch_bounds__(kBlock) k_heavy_keys(const float* __restrict__ est, int64_t d,
+                                                       const double* __restrict__ theta_p, uint64_t fill_seed,
+                                                       uint32_t* __restrict__ keys, uint32_t* hist1, SelectState* st,
+                                                       uint32_t k) {
+  __shared__ uint32_t sh[kBins];
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
+  __syncthreads();
+  const double theta = __ldcg(theta_p);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int lane = threadIdx.x & 31;
+  for (int64_t i0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < d; i0 += stride) {
+    const int64_t i = i0 + lane;
+    uint32_t bin = kNone;
+    if (i < d) {
+      const float e = est[i];
+      const double e2 = (double)e * (double)e;  // exact
+      const uint32_t key = e2 >= theta ? (0x80000000u | key_of(e))
+                                       : 0x7FFFFFFFu - (uint32_t)(splitmix64_at(fill_seed, (uint64_t)i) >> 33);
+      keys[i] = key;
+      bin = key >> kL1Shift;
+    }
+    hist_add(sh, bin);
+  }
+  hist_flush(sh, hist1, kBins);
+  last_block_pick(hist1, 11, st, 0, k);
+}
+
 // ---- launchers -----------------------------------------------------------------------------
 
 template <typename K>
@@ -697,6 +797,7 @@ QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, u
   qp.c = c;
   qp.cmask = c - 1;
   qp.vec = (reinterpret_cast<uintptr_t>(est) & 15u) == 0 ? 1 : 0;
+  qp.hist_on = 1;
   qp.h = h;
   return qp;
 }
@@ -745,22 +846,23 @@ size_t query_topk_workspace_bytes(int64_t d, int64_t k) {
          2 * align256((size_t)nbw * sizeof(uint32_t)) + align256((size_t)nblk * 4 * sizeof(uint32_t));
 }
 
-cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
-                              int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, cudaStream_t s) {
-  Workspace w = carve(workspace, d);
-  float* est = est_out ? est_out : w.est;
+namespace {
+
+// Histograms, state and both bitmaps back to zero.
+cudaError_t clear_selection(const Workspace& w, cudaStream_t s) {
   cudaError_t err = cudaMemsetAsync(w.hist, 0, 3 * kBins * sizeof(uint32_t), s);
   if (err == cudaSuccess) err = cudaMemsetAsync(w.st, 0, sizeof(SelectState), s);
   // the two bitmaps are adjacent: clear both at once
   if (err == cudaSuccess)
     err = cudaMemsetAsync(w.gt_bm, 0, (size_t)(reinterpret_cast<char*>(w.blk) - reinterpret_cast<char*>(w.gt_bm)), s);
-  if (err != cudaSuccess) return err;
+  return err;
+}
 
-  const QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
-  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
-  k_cand<<<persistent_grid(k_cand, (d + 3) / 4 / kU, kBlock), kBlock, 0, s>>>(est, d, qp.vec, w.st, w.hist + kBins,
-                                                                                 w.cand, w.gt_bm);
+// Levels 2 and 3 and the ordered output, after the level-1 histogram and pick of `src` keys.
+cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint32_t kmask, int64_t d, int64_t k,
+                             int64_t* idx_out, cudaStream_t s) {
+  k_cand<<<persistent_grid(k_cand, (d + 3) / 4 / kU, kBlock), kBlock, 0, s>>>(src, d, vec, kmask, w.st,
+                                                                                 w.hist + kBins, w.cand, w.gt_bm);
   const int small_grid = device_info().sms;
   k_cand_hist3<<<small_grid, kBlock, 0, s>>>(w.cand, w.st, w.hist + 2 * kBins);
   k_cand_mark<<<small_grid, kBlock, 0, s>>>(w.cand, w.st, w.gt_bm, w.eq_bm);
@@ -773,6 +875,50 @@ cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, u
   k_scan<<<1, kScanThreads, 0, s>>>(blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx);
   k_bm_write<<<nb, kBmThreads, 0, s>>>(w.gt_bm, w.eq_bm, w.nbw, w.st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
+                              int64_t d, int64_t k, int64_t* idx_out, float* est_out,
+                              void* workspace, cudaStream_t s) {
+  Workspace w = carve(workspace, d);
+  float* est = est_out ? est_out : w.est;
+  cudaError_t err = clear_selection(w, s);
+  if (err != cudaSuccess) return err;
+
+  const QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
+  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
+  return select_from_keys(w, est, qp.vec, 0x7FFFFFFFu, d, k, idx_out, s);
+}
+
+size_t heavymix_workspace_bytes(int64_t d, int64_t k) {
+  return query_topk_workspace_bytes(d, k) + align256((size_t)d * sizeof(uint32_t)) + 256;
+}
+
+cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
+                                  int64_t k, uint64_t fill_seed, int64_t* idx_out, float* est_out, double* l2sq_out,
+                                  void* workspace, cudaStream_t s) {
+  Workspace w = carve(workspace, d);
+  char* extra = static_cast<char*>(workspace) + query_topk_workspace_bytes(d, k);
+  uint32_t* keys = reinterpret_cast<uint32_t*>(extra);
+  double* sumsq = reinterpret_cast<double*>(extra + align256((size_t)d * sizeof(uint32_t)));
+  double* theta = sumsq + GS_MAX_ROWS;
+  float* est = est_out ? est_out : w.est;
+  cudaError_t err = clear_selection(w, s);
+  if (err == cudaSuccess) err = cudaMemsetAsync(sumsq, 0, 256, s);
+  if (err != cudaSuccess) return err;
+
+  QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
+  qp.hist_on = 0;
+  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
+  const int gx = (int)(((int64_t)c + kBlock - 1) / kBlock < 4 * device_info().sms ? ((int64_t)c + kBlock - 1) / kBlock
+                                                                                  : 4 * device_info().sms);
+  k_row_sumsq<<<dim3(gx, r), kBlock, 0, s>>>(merged, c, sumsq);
+  k_heavy_theta<<<1, 32, 0, s>>>(sumsq, r, k, theta, l2sq_out);
+  k_heavy_keys<<<persistent_grid(k_heavy_keys, d, kBlock), kBlock, 0, s>>>(est, d, theta, fill_seed, keys, w.hist,
+                                                                           w.st, (uint32_t)k);
+  return select_from_keys(w, reinterpret_cast<const float*>(keys), 1, 0xFFFFFFFFu, d, k, idx_out, s);
 }
 
 // ---- scratch without allocation ---------------------------------------------------------
@@ -834,8 +980,8 @@ cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, 
   const QueryParams qp = make_query_params(merged, h, r, c, d, k, est_out, hist, st);
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   const int hgrid = persistent_grid(k_hist, (d + 3) / 4 / kU, kBlock);
-  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + kBins, 9, 11, 1);
-  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + 2 * kBins, 0, 9, 2);
+  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + kBins, kL2Shift, 11, 1);
+  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + 2 * kBins, 0, kL3Bits, 2);
   const int nb = (int)nseg;
   if (qp.vec) k_count<true><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_gt, blk_eq);
   else k_count<false><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_gt, blk_eq);

@@ -350,3 +350,112 @@ def test_internal_estimate_query_matches(gs, H, r):
             H.check_vals(H.host(run.vals), idx, res.es_pre)
     finally:
         run.close()
+
+
+# ---- step 7: weight update (Alg. 1 step 26) ------------------------------------------------
+
+def test_apply_update_bit_exact(gs):
+    rng = np.random.default_rng(77)
+    d, k = 1_000_003, 5000
+    w = (rng.standard_normal(d) * 10.0 ** rng.integers(-5, 3, d)).astype(np.float32)
+    idx = np.sort(rng.choice(d, k, replace=False)).astype(np.int64)
+    vals = (rng.standard_normal(k) * 10.0 ** rng.integers(-8, 2, k)).astype(np.float32)
+    wd = _dev(w)
+    gs.gs_apply_update(wd, d, _dev(idx), _dev(vals), k, 0.03)
+    want = oracle.apply_update(w, idx, vals, 0.03)
+    assert np.array_equal(wd.cpu().numpy().view(np.uint32), want.view(np.uint32))
+    # indices outside [0, d) are skipped
+    w2 = _dev(np.ones(10, np.float32))
+    gs.gs_apply_update(w2, 10, _dev(np.array([-1, 3, 10], np.int64)), _dev(np.ones(3, np.float32)), 3, 1.0)
+    assert w2.cpu().numpy().tolist() == [1, 1, 1, 0, 1, 1, 1, 1, 1, 1]
+
+
+def test_gather_zero_update_fused(gs):
+    rng = np.random.default_rng(78)
+    P, d, k, lr = 6, 200_001, 777, 0.1
+    us = [(rng.standard_normal(d)).astype(np.float32) for _ in range(P)]
+    es = [(rng.standard_normal(d)).astype(np.float32) for _ in range(P)]
+    w = rng.standard_normal(d).astype(np.float32)
+    idx = np.sort(rng.choice(d, k, replace=False)).astype(np.int64)
+    ud, ed, wd = [_dev(u) for u in us], [_dev(e) for e in es], _dev(w)
+    vals = torch.empty(k, dtype=torch.float32, device="cuda")
+    gs.gs_gather_zero_update(ud, ed, d, _dev(idx), k, vals, wd, lr)
+    ref = np.zeros(k, np.float32)
+    for e in es:
+        ref = (ref + e[idx]).astype(np.float32)
+    assert np.array_equal(vals.cpu().numpy(), ref)
+    want = oracle.apply_update(w, idx, ref, lr)
+    assert np.array_equal(wd.cpu().numpy().view(np.uint32), want.view(np.uint32))
+    _, us2, es2 = oracle.gather_and_zero(us, es, idx)
+    for p in range(P):
+        assert np.array_equal(ud[p].cpu().numpy(), us2[p]) and np.array_equal(ed[p].cpu().numpy(), es2[p])
+
+
+def test_train_steps(gs, H):
+    """Alg. 1 end to end for the simulated workers: compression step plus weight update."""
+    w_cfg = workloads.get_config("resnet18")
+    P, d, r, c, k, seed, lr = 8, 250_001, 5, 1 << 12, 250, 17, 0.05
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w_cfg.rho)
+    try:
+        w = _dev(np.random.default_rng(3).standard_normal(d).astype(np.float32))
+        for t in range(3):
+            grads = workloads.make_gradients(w_cfg, t, range(P), d=d)
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            w0 = H.host(w)
+            gs.gs_train_step(run.sketch, w, lr, run.us, run.es, [_dev(g) for g in grads], d, w_cfg.rho, k, run.idx,
+                             run.vals, run.est, run.ws)
+            torch.cuda.synchronize()
+            res = oracle.step(us0, es0, grads, w_cfg.rho, coeffs, c, k)
+            idx, vals = H.host(run.idx), H.host(run.vals)
+            H.compare_step(res, coeffs, [H.host(u) for u in run.us], [H.host(e) for e in run.es], idx, vals,
+                           H.host(run.est), k)
+            want = oracle.apply_update(w0, idx, vals, lr)
+            assert np.array_equal(H.host(w).view(np.uint32), want.view(np.uint32))
+    finally:
+        run.close()
+
+
+# ---- HEAVYMIX (Alg. 2 as printed) ----------------------------------------------------------
+
+@pytest.mark.parametrize("d,r,c,k,spikes,scale", [(400_003, 5, 1 << 12, 300, 40, 50.0),
+                                                  (400_003, 5, 1 << 12, 5, 40, 50.0),
+                                                  (250_001, 4, 3001, 2000, 10, 20.0),
+                                                  (1 << 20, 7, 1 << 14, 1000, 5243, 100.0)])
+def test_heavymix(gs, H, d, r, c, k, spikes, scale):
+    seed, fill_seed = d % 1000 + r, 2**63 + 12345
+    rng = np.random.default_rng(seed)
+    x = (rng.standard_normal(d) * 1e-3).astype(np.float32)
+    x[rng.choice(d, spikes, replace=False)] *= np.float32(scale)
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(1, d, r, c, k, seed)
+    try:
+        gs.gs_sketch_insert(run.sketch, 0, _dev(x), d)
+        gs.gs_sketch_merge_tree(run.sketch, 1)
+        ws = torch.empty(gs.gs_query_heavymix_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        l2 = torch.empty(1, dtype=torch.float64, device="cuda")
+        gs.gs_query_heavymix(run.sketch, d, k, fill_seed, run.idx, run.est, l2, ws)
+        torch.cuda.synchronize()
+        idx, est, l2sq = H.host(run.idx), H.host(run.est), float(l2.item())
+        merged = H.merged_table(run, r, c).astype(np.float64)
+        rows = np.sort((merged ** 2).sum(axis=1))
+        want_l2 = rows[r // 2] if r % 2 else 0.5 * (rows[r // 2 - 1] + rows[r // 2])
+        assert abs(l2sq - want_l2) <= 1e-12 * want_l2
+        # exact: the selection rule applied to the GPU's own estimate and l2sq
+        assert np.array_equal(idx, oracle.heavymix_select(est, l2sq, k, fill_seed))
+        # against the fp64 oracle: the same l2sq within the cell tolerance, est within its band
+        T, A = oracle.sketch(x, coeffs, c)
+        idx_o, est_o, l2_o = oracle.heavymix(T, coeffs, d, k, fill_seed)
+        assert abs(l2sq - l2_o) <= 1e-4 * l2_o
+        band = oracle.cell_band(A, coeffs, np.arange(d))
+        assert np.all(np.abs(est.astype(np.float64) - est_o) <= band)
+        h_gpu = est.astype(np.float64) ** 2 >= l2sq / k
+        h_o = est_o.astype(np.float32).astype(np.float64) ** 2 >= l2_o / k
+        flip = np.nonzero(h_gpu != h_o)[0]
+        edge = np.abs(np.abs(est_o[flip]) - np.sqrt(l2_o / k)) <= band[flip] + 1e-4 * np.sqrt(l2_o / k)
+        assert np.all(edge), f"H differs away from the threshold at {flip[~edge][:5]}"
+        if flip.size == 0 and h_gpu.sum() < k:
+            assert np.array_equal(idx, idx_o)
+    finally:
+        run.close()

@@ -348,3 +348,101 @@ def test_step_output_contract():
         want = np.sum([e[res.idx].astype(np.float64) for e in res.es_pre], axis=0)
         assert np.array_equal(res.vals, want)
         us, es = res.us, res.es
+
+
+# ---- weight update -----------------------------------------------------------------------
+
+def test_apply_update_equals_numpy_fp32():
+    rng = np.random.default_rng(55)
+    d, k = 50_000, 700
+    w = (rng.standard_normal(d) * 10.0 ** rng.integers(-5, 3, d)).astype(np.float32)
+    idx = np.sort(rng.choice(d, k, replace=False))
+    vals = (rng.standard_normal(k) * 10.0 ** rng.integers(-8, 2, k)).astype(np.float32)
+    for lr in (0.1, 0.03, 1.0):
+        got = oracle.apply_update(w, idx, vals, lr)
+        want = w.copy()
+        want[idx] = w[idx] - np.float32(lr) * vals      # numpy fp32: two roundings, no fusion
+        assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+        mask = np.ones(d, bool)
+        mask[idx] = False
+        assert np.array_equal(got[mask], w[mask])
+
+
+def test_apply_update_closed_form():
+    w = np.full(8, 3.0, np.float32)
+    out = oracle.apply_update(w, [1, 5], np.array([2.0, -4.0], np.float32), 0.5)
+    assert out.tolist() == [3.0, 2.0, 3.0, 3.0, 3.0, 5.0, 3.0, 3.0]
+
+
+# ---- HEAVYMIX ----------------------------------------------------------------------------
+
+def test_splitmix64_counter_form_matches_stream():
+    lines = [l.strip() for l in open(os.path.join(GOLDEN, "splitmix64_seed1234567.txt"))
+             if l.strip() and not l.startswith("#")]
+    want = [int(x) for x in lines[1:]]
+    assert [int(v) for v in oracle.splitmix64_at(1234567, np.arange(5))] == want
+    for seed in (0, 99, 2**64 - 1):
+        gen = oracle.splitmix64(seed)
+        stream = [next(gen) for _ in range(50)]
+        assert [int(v) for v in oracle.splitmix64_at(seed, np.arange(50))] == stream
+
+
+def _heavymix_fixture(seed, d=600, r=5):
+    rng = np.random.default_rng(seed)
+    co = _injective_coeffs(r, seed)
+    x = _dyadic(rng, d, -64, 64, 2.0**-6)
+    x[rng.choice(d, 12, replace=False)] = np.float32(8.0)
+    T, _ = oracle.sketch(x, co, c=d)
+    return co, x, T
+
+
+def test_heavymix_l2_estimate_and_h():
+    co, x, T = _heavymix_fixture(1)
+    d, k = x.size, 20
+    idx, est, l2sq = oracle.heavymix(T, co, d, k, fill_seed=3)
+    assert np.array_equal(est, x.astype(np.float64))           # collision-free rows
+    assert l2sq == np.sum(x.astype(np.float64) ** 2)           # every row holds ||x||^2
+    spikes = np.nonzero(x == 8.0)[0]
+    assert set(spikes.tolist()) <= set(idx.tolist()) and idx.size == k
+
+
+def test_heavymix_h_bound_and_large_h_branch():
+    # with exact estimates sum_{i in H} x_i^2 >= |H| l2sq / k forces |H| <= k ...
+    rng = np.random.default_rng(6)
+    x = rng.standard_normal(2000)
+    for k in (1, 5, 50, 500):
+        h = x * x >= np.sum(x * x) / k
+        assert h.sum() <= k
+    # ... so |H| > k comes from estimation noise; with an underestimated l2sq, H is a
+    # superset of the top-k and the top-k of H by |est| is the plain top-k, ties by index
+    est = np.array([3.0, -5.0, 5.0, 1.0, 4.0, -4.0, 0.5])
+    idx = oracle.heavymix_select(est, l2sq=1.0, k=3, fill_seed=0)   # H = |est| >= 0.577...
+    assert idx.tolist() == [1, 2, 4]
+    assert np.array_equal(idx, oracle.topk(est, 3))
+
+
+def test_heavymix_random_fill_brute_force():
+    co, x, T = _heavymix_fixture(2)
+    d, k, seed = x.size, 200, 12345
+    idx, est, l2sq = oracle.heavymix(T, co, d, k, fill_seed=seed)
+    h = [i for i in range(d) if float(x[i]) ** 2 >= l2sq / k]
+    assert len(h) < k
+    xi = {i: int(oracle.splitmix64_at(seed, [i])[0]) >> 33 for i in range(d)}
+    nh = sorted((i for i in range(d) if i not in set(h)), key=lambda i: (xi[i], i))
+    assert sorted(h + nh[: k - len(h)]) == idx.tolist()
+
+
+def test_heavymix_fill_is_uniform():
+    co, x, T = _heavymix_fixture(4, d=300)
+    d, k = x.size, 60
+    counts = np.zeros(d)
+    trials = 400
+    for seed in range(trials):
+        idx, _, l2sq = oracle.heavymix(T, co, d, k, fill_seed=seed)
+        counts[idx] += 1
+    in_h = x.astype(np.float64) ** 2 >= l2sq / k
+    assert np.all(counts[in_h] == trials)
+    nh = ~in_h
+    p = (k - in_h.sum()) / nh.sum()
+    z = (counts[nh] - trials * p) / np.sqrt(trials * p * (1 - p))
+    assert abs(z.mean()) < 0.2 and np.max(np.abs(z)) < 5.0
