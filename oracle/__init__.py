@@ -46,6 +46,10 @@ from .gssgd import (  # noqa: F401
     heavymix_select,
     gather_and_zero,
     apply_update,
+    query_at,
+    sketch_sparse,
+    sketched_state_step,
+    SketchedStateResult,
     step,
     StepResult,
 )

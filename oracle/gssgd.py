@@ -218,6 +218,82 @@ def apply_update(w: np.ndarray, idx, vals, lr: float) -> np.ndarray:
     return w2
 
 
+# ---- 8. momentum and error kept as sketches ----------------------------------------------
+
+def query_at(T: np.ndarray, coeffs, idx) -> np.ndarray:
+    """The median estimate of ``query`` at the coordinates ``idx`` only (fp64)."""
+    idx = np.asarray(idx, dtype=np.uint64)
+    c = T.shape[1]
+    buckets, signs = hash_rows(coeffs, c, idx)
+    r = buckets.shape[0]
+    vals = np.stack([signs[j] * T[j][buckets[j]] for j in range(r)]).astype(np.float64)
+    vals.sort(axis=0)
+    if r % 2 == 1:
+        return vals[r // 2].copy()
+    return 0.5 * (vals[r // 2 - 1] + vals[r // 2])
+
+
+def sketch_sparse(idx, vals, coeffs, c: int):
+    """(T, A): the Count Sketch of the sparse vector with vals at idx (fp64), and its
+    magnitude table."""
+    idx = np.asarray(idx, dtype=np.uint64)
+    v = np.asarray(vals, dtype=np.float64)
+    buckets, signs = hash_rows(coeffs, c, idx)
+    r = buckets.shape[0]
+    T = np.zeros((r, c))
+    A = np.zeros((r, c))
+    for j in range(r):
+        T[j] = np.bincount(buckets[j], weights=signs[j] * v, minlength=c)
+        A[j] = np.bincount(buckets[j], weights=np.abs(v), minlength=c)
+    return T, A
+
+
+@dataclasses.dataclass
+class SketchedStateResult:
+    S: np.ndarray       # merged sketch of the step's gradients
+    U: np.ndarray       # momentum sketch after the step
+    E: np.ndarray       # error sketch after the step
+    AU: np.ndarray      # magnitude tables of U and E (tolerance bands)
+    AE: np.ndarray
+    est: np.ndarray     # estimate from the accumulated error sketch (before removal)
+    band: np.ndarray    # per-coordinate band of est
+    idx: np.ndarray     # selected coordinates, ascending
+    delta: np.ndarray   # values sent for the update: the error sketch's estimate at idx
+    delta_u: np.ndarray # the momentum sketch's estimate at idx (removed from U)
+    U_pre: np.ndarray   # U and E after accumulation, before the removal
+    E_pre: np.ndarray
+    AU_pre: np.ndarray
+    AE_pre: np.ndarray
+    AS: np.ndarray      # magnitude table of S
+
+
+def sketched_state_step(U, E, AU, AE, gs, rho: float, coeffs, c: int, k: int, rel: float = 1e-5):
+    """One step with momentum and error carried as r x c sketches (the linear-sketch variant
+    named in Sec. II): S = tree merge of S(g_p); U <- rho U + S; E <- E + U; I = top-k of the
+    estimate from E; delta = that estimate at I; then the extracted mass leaves both sketches,
+    E <- E - S(delta), U <- U - S(delta_u) with delta_u the estimate of U at I.  fp64; AU, AE
+    carry the magnitude tables for the tolerance bands."""
+    d = np.asarray(gs[0]).size
+    hashes = hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+    sk = [sketch(g, coeffs, c, hashes) for g in gs]
+    S = merge_tree([t for t, _ in sk])
+    AS = merge_tree([a for _, a in sk])
+    r64 = np.float64(np.float32(rho))
+    U1 = r64 * np.asarray(U, np.float64) + S
+    AU1 = r64 * np.asarray(AU, np.float64) + AS
+    E1 = np.asarray(E, np.float64) + U1
+    AE1 = np.asarray(AE, np.float64) + AU1
+    est = query(E1, coeffs, d, hashes)
+    band = cell_band(AE1, coeffs, np.arange(d), rel)
+    idx = topk(est, k)
+    delta = est[idx]
+    delta_u = query_at(U1, coeffs, idx)
+    SD, AD = sketch_sparse(idx, delta, coeffs, c)
+    SDu, ADu = sketch_sparse(idx, delta_u, coeffs, c)
+    return SketchedStateResult(S, U1 - SDu, E1 - SD, AU1 + ADu, AE1 + AD, est, band, idx, delta, delta_u,
+                               U1, E1, AU1, AE1, AS)
+
+
 # ---- one full step ---------------------------------------------------------------------
 
 @dataclasses.dataclass

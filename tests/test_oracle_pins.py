@@ -446,3 +446,51 @@ def test_heavymix_fill_is_uniform():
     p = (k - in_h.sum()) / nh.sum()
     z = (counts[nh] - trials * p) / np.sqrt(trials * p * (1 - p))
     assert abs(z.mean()) < 0.2 and np.max(np.abs(z)) < 5.0
+
+
+# ---- momentum and error kept as sketches -------------------------------------------------
+
+def test_sketch_sparse_is_sketch_of_dense():
+    rng = np.random.default_rng(61)
+    d, r, c = 3000, 5, 256
+    co = oracle.derive_coefficients(r, 61)
+    idx = np.sort(rng.choice(d, 40, replace=False))
+    vals = _dyadic(rng, 40)
+    dense = np.zeros(d, np.float32)
+    dense[idx] = vals
+    T, A = oracle.sketch_sparse(idx, vals, co, c)
+    T2, A2 = oracle.sketch(dense, co, c)
+    assert np.array_equal(T, T2) and np.array_equal(A, A2)
+    assert np.array_equal(oracle.query_at(T, co, idx), oracle.query(T, co, d)[idx])
+
+
+def test_sketched_state_removal_and_momentum_closed_form():
+    # collision-free rows: every estimate is exact, so after the step the selected
+    # coordinates read exactly 0 in both sketches and everything else is untouched
+    rng = np.random.default_rng(62)
+    d, r, k, P = 500, 3, 20, 4
+    co = _injective_coeffs(r, 62)
+    zeros = np.zeros((r, d))
+    gs = [_dyadic(rng, d, -64, 64, 2.0**-6) for _ in range(P)]
+    res = oracle.sketched_state_step(zeros, zeros, zeros, zeros, gs, 0.5, co, d, k)
+    total = np.sum(np.stack(gs).astype(np.float64), axis=0)
+    assert np.array_equal(res.est, total)          # U = S, E = U after the first step
+    assert np.array_equal(res.idx, oracle.topk(total, k))
+    assert np.array_equal(res.delta, total[res.idx])
+    assert np.all(oracle.query_at(res.E, co, res.idx) == 0)
+    assert np.all(oracle.query_at(res.U, co, res.idx) == 0)
+    rest = np.setdiff1d(np.arange(d), res.idx)
+    assert np.array_equal(oracle.query_at(res.E, co, rest), total[rest])
+    # momentum/error recursion, rho = 1/2, g = 1/4 everywhere, k = 1: step t takes
+    # coordinate t - 1 (all remaining ones tie and the smaller index wins), and every
+    # coordinate not yet taken follows U_t = (2 - 2^(1-t))/4, E_t = (2t - 2 + 2^(1-t))/4
+    g = [np.full(d, 0.25, np.float32)]
+    U = E = AU = AE = np.zeros((r, d))
+    for t in range(1, 6):
+        res = oracle.sketched_state_step(U, E, AU, AE, g, 0.5, co, d, 1)
+        U, E, AU, AE = res.U, res.E, res.AU, res.AE
+        assert res.idx.tolist() == [t - 1]
+        rest = np.arange(t, d)
+        assert np.all(oracle.query_at(U, co, rest) == (2 - 2.0 ** (1 - t)) / 4)
+        assert np.all(oracle.query_at(E, co, rest) == (2 * t - 2 + 2.0 ** (1 - t)) / 4)
+        assert oracle.query_at(E, co, [t - 1])[0] == 0 and oracle.query_at(U, co, [t - 1])[0] == 0
