@@ -344,7 +344,8 @@ def run_ours(args):
         cpu = cpu_baseline(w, steps=2)
 
     gs.gs_sketch_destroy(sk)
-    launches_per_step = groups + 1 + 9 + 1  # insert groups, merge, query/top-k (9), gather
+    # fused insert (one per group and row pass), merge, query + selection (7), gather
+    launches_per_step = groups * passes + 1 + 7 + 1
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4), "higher_is_better": True,

@@ -234,6 +234,42 @@ gs_status gs_train_step(gs_sketch* sketch, float* weights, float lr, float* cons
                         int64_t k, int64_t* idx_out, float* vals_out, float* est_out,
                         void* workspace, size_t workspace_bytes, gs_stream stream);
 
+/* ---- momentum and error kept as sketches ------------------------------------------ */
+/* Sec. II notes that a linear sketch can carry momentum and error accumulation itself.  In
+ * this variant the state is two r x c tables instead of 2P vectors of length d: the
+ * merged tables of two sketches `momentum` (U) and `error` (E) created with the same r, c
+ * and seed as the workers' sketch set (any worker count; only their merged tables are used,
+ * and they start at zero). */
+
+/* Device pointer of a sketch's merged table (fp32 [r][c], library-owned). */
+gs_status gs_sketch_merged_table(const gs_sketch* sketch, float** table_out);
+
+/* est_out[t] = median over rows j of s_j(idx[t]) * T[j][h_j(idx[t])] on the merged table,
+ * for k coordinates (the query of Alg. 2 step 1 at given indices). */
+gs_status gs_sketch_query_at(const gs_sketch* sketch, const int64_t* idx, int64_t k,
+                             float* est_out, gs_stream stream);
+
+/* merged[j][h_j(idx[t])] += scale * s_j(idx[t]) * vals[t] for every row and t < k: adds
+ * scale * S(v) for the sparse vector v with vals at idx (fp32 atomic additions). */
+gs_status gs_sketch_add_sparse(gs_sketch* sketch, const int64_t* idx, const float* vals,
+                               int64_t k, float scale, gs_stream stream);
+
+/* One step with sketched momentum and error:
+ *   S = tree merge of S(grad[p]) over the workers' sketch set (steps 2-3 on raw gradients);
+ *   U <- fl(fl(rho U) + S), E <- fl(E + U)           elementwise on the r*c cells;
+ *   idx_out = the top-k of the estimate from E        (as gs_query_topk on E);
+ *   vals_out = that estimate at idx_out                (delta; no per-coordinate exact
+ *                                                      values exist in this variant);
+ *   E <- E - S(delta), U <- U - S(delta_u), delta_u = the estimate from U at idx_out
+ *                                                      (the extracted mass leaves both);
+ *   weights (nullable) <- weights - lr * delta at idx_out.
+ * workspace: gs_step_workspace_size(d, k) bytes.  GS_ERR_MISMATCH unless the three sketches
+ * share r, c and seed. */
+gs_status gs_sketched_state_step(gs_sketch* workers, gs_sketch* momentum, gs_sketch* error,
+                                 const float* const* grad, int64_t d, float rho, int64_t k,
+                                 int64_t* idx_out, float* vals_out, float* weights, float lr,
+                                 void* workspace, size_t workspace_bytes, gs_stream stream);
+
 /* gs_step with the gradients in HOST memory and the results returned to HOST memory, one
  * synchronous call per step.  Where the device can address grad_host[p] in place (memory
  * from cudaHostAlloc or cudaHostRegister, or any host memory on systems whose GPU has

@@ -53,6 +53,10 @@ SIGNATURES = {
     "gs_apply_update": [_vp, _i64, _vp, _vp, _i64, _f32, _vp],
     "gs_gather_zero_update": [_PP, _PP, _i32, _i64, _vp, _i64, _vp, _vp, _f32, _vp],
     "gs_train_step": [_vp, _vp, _f32, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
+    "gs_sketch_merged_table": [_vp, ctypes.POINTER(_vp)],
+    "gs_sketch_query_at": [_vp, _vp, _i64, _vp, _vp],
+    "gs_sketch_add_sparse": [_vp, _vp, _vp, _i64, _f32, _vp],
+    "gs_sketched_state_step": [_vp, _vp, _vp, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _f32, _vp, _sz, _vp],
     "gs_step_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_step": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
     "gs_step_host": [_vp, _PP, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _sz, _vp],
@@ -230,6 +234,31 @@ def gs_train_step(sketch: int, weights, lr: float, momentum, error, grad, d: int
     _check(load_library().gs_train_step(sketch, _ptr(weights), lr, _ptr_array(momentum), _ptr_array(error),
                                         _ptr_array(grad), d, rho, k, _ptr(idx_out), _ptr(vals_out), _ptr(est_out),
                                         _ptr(workspace), workspace_bytes, _stream(stream)), "gs_train_step")
+
+
+def gs_sketch_merged_table(sketch: int) -> int:
+    out = _vp()
+    _check(load_library().gs_sketch_merged_table(sketch, ctypes.byref(out)), "gs_sketch_merged_table")
+    return out.value
+
+
+def gs_sketch_query_at(sketch: int, idx, k: int, est_out, stream=None) -> None:
+    _check(load_library().gs_sketch_query_at(sketch, _ptr(idx), k, _ptr(est_out), _stream(stream)),
+           "gs_sketch_query_at")
+
+
+def gs_sketch_add_sparse(sketch: int, idx, vals, k: int, scale: float, stream=None) -> None:
+    _check(load_library().gs_sketch_add_sparse(sketch, _ptr(idx), _ptr(vals), k, scale, _stream(stream)),
+           "gs_sketch_add_sparse")
+
+
+def gs_sketched_state_step(workers: int, momentum: int, error: int, grad, d: int, rho: float, k: int, idx_out,
+                           vals_out, weights, lr: float, workspace, workspace_bytes=None, stream=None) -> None:
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(load_library().gs_sketched_state_step(workers, momentum, error, _ptr_array(grad), d, rho, k, _ptr(idx_out),
+                                                 _ptr(vals_out), _ptr(weights), lr, _ptr(workspace), workspace_bytes,
+                                                 _stream(stream)), "gs_sketched_state_step")
 
 
 def gs_step_workspace_size(d: int, k: int) -> int:

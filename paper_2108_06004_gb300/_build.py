@@ -19,7 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libgs_sketch.so")
-SOURCES = ["gs_api.cu", "k_insert.cu", "k_merge.cu", "k_query_topk.cu", "k_gather.cu"]
+SOURCES = ["gs_api.cu", "k_insert.cu", "k_merge.cu", "k_query_topk.cu", "k_gather.cu", "k_sketch_state.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xptxas", "-v",
                  "-I", INCLUDE, "-I", CSRC]

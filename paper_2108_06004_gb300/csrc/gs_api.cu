@@ -162,6 +162,40 @@ gs_status accumulate_insert_impl(gs_sketch* sk, int32_t first, int32_t n, float*
   return GS_OK;
 }
 
+// Insert the vectors vec[p] (no accumulation) into the worker tables, all groups and passes.
+gs_status insert_all_impl(gs_sketch* sk, const float* const* vec, int64_t d, cudaStream_t s) {
+  const int W = sk->W;
+  for (int grp = 0; grp * W < sk->workers; ++grp) {
+    gs::InsertParams p;
+    std::memset(&p, 0, sizeof(p));
+    const int lo = grp * W;
+    const int nw = (sk->workers - lo) < W ? (sk->workers - lo) : W;
+    bool vec_ok = true;
+    for (int w = 0; w < nw; ++w) {
+      p.e[w] = const_cast<float*>(vec[lo + w]);
+      vec_ok = vec_ok && aligned(vec[lo + w], 16);
+    }
+    p.table = sk->tables + (size_t)grp * sk->r * sk->c * W;
+    p.d = d;
+    p.nw = nw;
+    p.r = sk->r;
+    p.c = (uint32_t)sk->c;
+    p.cmask = (uint32_t)sk->c - 1;
+    p.h = sk->h;
+    for (int j0 = 0; j0 < sk->r; j0 += sk->rows_per_pass) {
+      p.j0 = j0;
+      p.j1 = (j0 + sk->rows_per_pass < sk->r) ? j0 + sk->rows_per_pass : sk->r;
+      cudaError_t err = gs::launch_accumulate_insert(p, W, false, vec_ok, s);
+      if (err != cudaSuccess) return cuda_fail(err, "insert launch");
+    }
+  }
+  return GS_OK;
+}
+
+bool same_family(const gs_sketch* a, const gs_sketch* b) {
+  return a->r == b->r && a->c == b->c && a->seed == b->seed;
+}
+
 gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float* const* g,
                     int64_t d, float rho, int64_t k, int64_t* idx, float* vals, float* est,
                     void* ws, cudaStream_t s, float* weights = nullptr, float lr = 0.f) {
@@ -586,6 +620,95 @@ gs_status gs_train_step(gs_sketch* sk, float* weights, float lr, float* const* m
   if (workspace_bytes < gs::query_topk_workspace_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small");
   return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, est_out, workspace, as_stream(stream),
                    weights, lr);
+  GS_GUARD_END
+}
+
+gs_status gs_sketch_merged_table(const gs_sketch* sk, float** table_out) {
+  if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
+  if (!table_out) return fail(GS_ERR_INVALID_ARG, "table_out is NULL");
+  *table_out = sk->merged;
+  return GS_OK;
+}
+
+gs_status gs_sketch_query_at(const gs_sketch* sk, const int64_t* idx, int64_t k, float* est_out, gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  if (k < 1) return fail(GS_ERR_INVALID_ARG, "k must be positive");
+  if (!idx || !aligned(idx, 8)) return fail(GS_ERR_INVALID_ARG, "idx is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(est_out, "est_out"));
+  cudaError_t e = gs::launch_query_at(sk->merged, sk->h, sk->r, (uint32_t)sk->c, idx, k, est_out, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "query_at launch");
+  return GS_OK;
+}
+
+gs_status gs_sketch_add_sparse(gs_sketch* sk, const int64_t* idx, const float* vals, int64_t k, float scale,
+                               gs_stream stream) {
+  GS_TRY(check_sketch(sk));
+  if (k < 1) return fail(GS_ERR_INVALID_ARG, "k must be positive");
+  if (!idx || !aligned(idx, 8)) return fail(GS_ERR_INVALID_ARG, "idx is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals, "vals"));
+  cudaError_t e = gs::launch_add_sparse(sk->merged, sk->h, sk->r, (uint32_t)sk->c, idx, vals, k, scale,
+                                        as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "add_sparse launch");
+  return GS_OK;
+}
+
+gs_status gs_sketched_state_step(gs_sketch* workers, gs_sketch* momentum, gs_sketch* error, const float* const* grad,
+                                 int64_t d, float rho, int64_t k, int64_t* idx_out, float* vals_out, float* weights,
+                                 float lr, void* workspace, size_t workspace_bytes, gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(workers));
+  GS_TRY(check_sketch(momentum));
+  GS_TRY(check_sketch(error));
+  if (!same_family(workers, momentum) || !same_family(workers, error))
+    return fail(GS_ERR_MISMATCH, "the three sketches must share r, c and seed");
+  if (momentum == error || momentum == workers || error == workers)
+    return fail(GS_ERR_INVALID_ARG, "workers, momentum and error must be three different sketches");
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  for (int p = 0; p < workers->workers; ++p) GS_TRY(check_vec(grad[p], "grad[p]"));
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals_out, "vals_out"));
+  if (weights) GS_TRY(check_vec(weights, "weights"));
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < step_ws_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_step_workspace_size");
+  cudaStream_t s = as_stream(stream);
+  const int64_t cells = (int64_t)workers->r * workers->c;
+  // S = tree merge of S(g_p)
+  const size_t tbytes = ((size_t)workers->groups * workers->r * workers->c * workers->W + (size_t)cells) * sizeof(float);
+  cudaError_t err = cudaMemsetAsync(workers->tables, 0, tbytes, s);
+  if (err != cudaSuccess) return cuda_fail(err, "zero tables");
+  GS_TRY(insert_all_impl(workers, grad, d, s));
+  gs::MergeParams mp;
+  mp.tables = workers->tables;
+  mp.merged = workers->merged;
+  mp.cells = cells;
+  mp.group_stride = cells * workers->W;
+  mp.P = workers->workers;
+  if ((err = gs::launch_merge(mp, workers->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
+  // U <- rho U + S ; E <- E + U   (elementwise on the r*c cells)
+  if ((err = gs::launch_accumulate(momentum->merged, error->merged, workers->merged, cells, rho, s)) != cudaSuccess)
+    return cuda_fail(err, "sketch accumulate launch");
+  // top-k of the estimate from E; delta = that estimate at the selected coordinates
+  if ((err = gs::launch_query_topk(error->merged, error->h, error->r, (uint32_t)error->c, d, k, idx_out, nullptr,
+                                   workspace, s)) != cudaSuccess)
+    return cuda_fail(err, "query/top-k launch");
+  const float* est = static_cast<const float*>(workspace);  // the query keeps est at the workspace start
+  if ((err = gs::launch_take(est, d, idx_out, k, vals_out, s)) != cudaSuccess) return cuda_fail(err, "take launch");
+  float* delta_u = reinterpret_cast<float*>(static_cast<char*>(workspace) + gs::query_topk_workspace_bytes(d, k));
+  if ((err = gs::launch_query_at(momentum->merged, momentum->h, momentum->r, (uint32_t)momentum->c, idx_out, k,
+                                 delta_u, s)) != cudaSuccess)
+    return cuda_fail(err, "query_at launch");
+  // the extracted mass leaves both sketches
+  if ((err = gs::launch_add_sparse(error->merged, error->h, error->r, (uint32_t)error->c, idx_out, vals_out, k, -1.f,
+                                   s)) != cudaSuccess)
+    return cuda_fail(err, "add_sparse launch");
+  if ((err = gs::launch_add_sparse(momentum->merged, momentum->h, momentum->r, (uint32_t)momentum->c, idx_out, delta_u,
+                                   k, -1.f, s)) != cudaSuccess)
+    return cuda_fail(err, "add_sparse launch");
+  if (weights && (err = gs::launch_apply_update(weights, d, idx_out, vals_out, k, lr, s)) != cudaSuccess)
+    return cuda_fail(err, "update launch");
+  return GS_OK;
   GS_GUARD_END
 }
 

@@ -123,6 +123,13 @@ cudaError_t launch_apply_update(float* w, int64_t d, const int64_t* idx, const f
                                 cudaStream_t s);
 
 size_t query_topk_workspace_bytes(int64_t d, int64_t k);
+
+// momentum and error kept as sketches
+cudaError_t launch_query_at(const float* T, const HashCoeffs& h, int r, uint32_t c, const int64_t* idx, int64_t k,
+                            float* out, cudaStream_t s);
+cudaError_t launch_add_sparse(float* T, const HashCoeffs& h, int r, uint32_t c, const int64_t* idx, const float* vals,
+                              int64_t k, float scale, cudaStream_t s);
+cudaError_t launch_take(const float* src, int64_t n, const int64_t* idx, int64_t k, float* out, cudaStream_t s);
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
                               void* workspace, cudaStream_t s);
