@@ -42,6 +42,16 @@ REF_BUDGET_S = 120.0     # oracle seconds for a whole --impl reference run
 ORACLE_S_PER_COORD = 1.7e-7  # oracle seconds per worker-coordinate (sizes the reference samples)
 
 
+VARIANTS = {
+    "error_feedback": "S1-S6: per-worker momentum and error vectors, exact second round",
+    "train": "S1-S7: as error_feedback, with the weight update fused into the second round",
+    "heavymix": "S1-S6 with the HEAVYMIX selection in place of the top-k",
+    "sketched_state": "momentum and error kept as r x c sketches; no per-worker state vectors",
+}
+HEAVYMIX_FILL_SEED = 0x5EED5EED
+LR = 0.01
+
+
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -49,6 +59,8 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="resnet18", choices=sorted(workloads.CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--variant", default="error_feedback", choices=list(VARIANTS),
+                    help="which form of the step to time (the default is the headline path)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-steps", action="store_true",
@@ -224,8 +236,20 @@ def run_ours(args):
     sk = gs.gs_sketch_create(r, c, 20210813, P, 0)
     W = gs.gs_sketch_info(sk)["group_width"]
     groups = (P + W - 1) // W
-    ws = torch.empty(gs.gs_step_workspace_size(d, k), dtype=torch.uint8, device=dev)
+    variant = args.variant
+    ws_bytes = gs.gs_step_workspace_size(d, k)
+    if variant == "heavymix":
+        ws_bytes = max(ws_bytes, gs.gs_query_heavymix_workspace_size(d, k))
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
     qws_bytes = gs.gs_query_topk_workspace_size(d, k)
+    l2sq = torch.empty(1, dtype=torch.float64, device=dev)
+    weights = torch.zeros(d, dtype=torch.float32, device=dev) if variant in ("train", "sketched_state") else None
+    sk_u = sk_e = None
+    if variant == "sketched_state":
+        sk_u = gs.gs_sketch_create(r, c, 20210813, 1, 0)
+        sk_e = gs.gs_sketch_create(r, c, 20210813, 1, 0)
+        gs.gs_sketch_zero(sk_u)
+        gs.gs_sketch_zero(sk_e)
     idx = torch.empty(k, dtype=torch.int64, device=dev)
     vals = torch.empty(k, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
@@ -235,6 +259,17 @@ def run_ours(args):
 
     def step(t, record):
         grads = dev_pool[t % nsteps_pool]
+        if variant == "sketched_state":
+            # one composed call; its whole duration is the timed unit
+            if record:
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            gs.gs_sketched_state_step(sk, sk_u, sk_e, grads, d, rho, k, idx, vals, weights, LR, ws, None, stream)
+            if record:
+                e1.record(stream)
+                k1_events.append((e0, e1, P))
+            return
         gs.gs_sketch_zero(sk, stream)
         for g0 in range(0, P, W):
             if record:
@@ -246,8 +281,14 @@ def run_ours(args):
                 e1.record(stream)
                 k1_events.append((e0, e1, min(W, P - g0)))
         gs.gs_sketch_merge_tree(sk, P, stream)
-        gs.gs_query_topk(sk, d, k, idx, None, ws, qws_bytes, stream)
-        gs.gs_gather_and_zero(us, es, d, idx, k, vals, stream)
+        if variant == "heavymix":
+            gs.gs_query_heavymix(sk, d, k, HEAVYMIX_FILL_SEED, idx, None, l2sq, ws, None, stream)
+        else:
+            gs.gs_query_topk(sk, d, k, idx, None, ws, qws_bytes, stream)
+        if variant == "train":
+            gs.gs_gather_zero_update(us, es, d, idx, k, vals, weights, LR, stream)
+        else:
+            gs.gs_gather_and_zero(us, es, d, idx, k, vals, stream)
 
     for t in range(args.warmup):
         step(t, False)
@@ -297,24 +338,32 @@ def run_ours(args):
     k1_gbs = (sum(k1_bytes) / len(k1_bytes)) / k1_avg_s / 1e9
     full_launch_bytes = per_wc * W * d
     reds_per_launch = d * r * ((W + 3) // 4)
+    if variant == "sketched_state":
+        # the timed unit is the whole composed call: read g once per row pass (4 B per
+        # worker-coordinate and pass), write and re-read the estimate (8 B per coordinate)
+        per_wc = 4.0 * passes
+        full_launch_bytes = per_wc * P * d + 8.0 * d
+        k1_gbs = full_launch_bytes / k1_avg_s / 1e9
     roofline = {
-        "kernel": "k_accumulate_insert (fused S1+S2), one call = one group of workers, all row passes",
+        "kernel": "gs_sketched_state_step (whole composed call)" if variant == "sketched_state" else
+                  "k_accumulate_insert (fused S1+S2), one call = one group of workers, all row passes",
         "row_passes": passes, "algorithmic_bytes_per_worker_coord": per_wc,
         "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
         "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
-        "traffic": k1_traffic_per_launch(),
+        "traffic": k1_traffic_per_launch() if variant != "sketched_state" else None,
         "algorithmic_bytes_per_launch": full_launch_bytes,
         "avg_launch_ms": round(sum(k1_ms) / len(k1_ms), 4),
         "co_bound": {"kind": "l2_reductions, 16-byte requests merged per 32-byte cell",
-                     "cell_updates_per_launch": d * r,
-                     "achieved_G_cells_per_s": round(d * r / k1_avg_s / 1e9, 1),
+                     "cell_updates_per_launch": d * r * (groups if variant == "sketched_state" else 1),
+                     "achieved_G_cells_per_s": round(d * r * (groups if variant == "sketched_state" else 1)
+                                                     / k1_avg_s / 1e9, 1),
                      "probe_peak_G_cells_per_s": 134.5},
         "step_share": round(sum(k1_ms) / elapsed_ms, 3),
     }
 
     # end to end through the public call with host buffers
     e2e = None
-    if not args.no_e2e and not args.profile_steps:
+    if not args.no_e2e and not args.profile_steps and variant == "error_feedback":
         grad_dev = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(P)]
         idx_h = torch.empty(k, dtype=torch.int64).pin_memory()
         vals_h = torch.empty(k, dtype=torch.float32).pin_memory()
@@ -340,17 +389,23 @@ def run_ours(args):
                "call": "gs_step_host"}
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_steps:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_steps \
+            and variant == "error_feedback":
         cpu = cpu_baseline(w, steps=2)
 
     gs.gs_sketch_destroy(sk)
-    # fused insert (one per group and row pass), merge, query + selection (7), gather
-    launches_per_step = groups * passes + 1 + 7 + 1
+    for extra in (sk_u, sk_e):
+        if extra:
+            gs.gs_sketch_destroy(extra)
+    # insert (one per group and row pass), merge, query + selection (7; HEAVYMIX 10), then
+    # the gather (sketched state: cell accumulate, take, query_at, two sparse inserts, update)
+    launches_per_step = groups * passes + 1 + (10 if variant == "heavymix" else 7) + \
+        (6 if variant == "sketched_state" else 1)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": w.name, "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
+        "config": {"workload": w.name, "variant": variant, "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
                    "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
                    "l2": f"inputs larger than L2 ({P * d * 12 / 1e9:.2f} GB of g,u,e streamed per step)",
                    "d_steps_per_s": world * d * args.steps / (elapsed_ms / 1e3)},
