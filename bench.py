@@ -61,6 +61,8 @@ def parse_args():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--variant", default="error_feedback", choices=list(VARIANTS),
                     help="which form of the step to time (the default is the headline path)")
+    ap.add_argument("--eager", action="store_true",
+                    help="one library call per kernel instead of a captured plan per step")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-steps", action="store_true",
@@ -255,31 +257,38 @@ def run_ours(args):
     stream = torch.cuda.current_stream()
     torch.cuda.synchronize()
 
+    # Plans (one CUDA graph per gradient buffer set, the insert phase timed by event nodes
+    # inside the graph) unless --eager asks for one library call per kernel.  HEAVYMIX has
+    # no plan form and always runs eagerly; the sketched state always runs as a plan.
+    use_plan = (not args.eager or variant == "sketched_state") and variant != "heavymix"
+    plans = []
+    if use_plan:
+        for grads in dev_pool:
+            if variant == "sketched_state":
+                plans.append(gs.gs_sketched_state_plan_create(sk, sk_u, sk_e, grads, d, rho, k, idx, vals, weights,
+                                                              LR, ws, flags=gs.GS_PLAN_TIME_INSERT))
+            else:
+                plans.append(gs.gs_step_plan_create(sk, us, es, grads, d, rho, k, idx, vals, None, weights, LR, ws,
+                                                    flags=gs.GS_PLAN_TIME_INSERT))
     k1_events = []
 
     def step(t, record):
+        if use_plan:
+            gs.gs_plan_launch(plans[t % nsteps_pool], stream)
+            return
         grads = dev_pool[t % nsteps_pool]
         if variant == "sketched_state":
-            # one composed call; its whole duration is the timed unit
-            if record:
-                e0 = torch.cuda.Event(enable_timing=True)
-                e1 = torch.cuda.Event(enable_timing=True)
-                e0.record(stream)
             gs.gs_sketched_state_step(sk, sk_u, sk_e, grads, d, rho, k, idx, vals, weights, LR, ws, None, stream)
-            if record:
-                e1.record(stream)
-                k1_events.append((e0, e1, P))
             return
         gs.gs_sketch_zero(sk, stream)
-        for g0 in range(0, P, W):
-            if record:
-                e0 = torch.cuda.Event(enable_timing=True)
-                e1 = torch.cuda.Event(enable_timing=True)
-                e0.record(stream)
-            gs.gs_accumulate_insert(sk, g0, us[g0:g0 + W], es[g0:g0 + W], grads[g0:g0 + W], d, rho, stream)
-            if record:
-                e1.record(stream)
-                k1_events.append((e0, e1, min(W, P - g0)))
+        if record:
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        gs.gs_accumulate_insert(sk, 0, us, es, grads, d, rho, stream)
+        if record:
+            e1.record(stream)
+            k1_events.append((e0, e1))
         gs.gs_sketch_merge_tree(sk, P, stream)
         if variant == "heavymix":
             gs.gs_query_heavymix(sk, d, k, HEAVYMIX_FILL_SEED, idx, None, l2sq, ws, None, stream)
@@ -321,72 +330,94 @@ def run_ours(args):
     if sampler:
         clocks = sampler.stop()
 
-    k1_ms = [a.elapsed_time(b) for a, b, _ in k1_events]
-    k1_lanes = [n for _, _, n in k1_events]
-    coords = world * P * d * args.steps
+    # insert-phase durations of the timed steps: each covers all groups and row passes
+    if use_plan:
+        k1_ms = []
+        for i, plan in enumerate(plans):
+            n_timed = sum(1 for t in range(args.steps) if (args.warmup + t) % nsteps_pool == i)
+            if n_timed:
+                k1_ms += gs.gs_plan_insert_times(plan, n_timed)
+    else:
+        k1_ms = [a.elapsed_time(b) for a, b in k1_events]
     value = whole_job_rate(world, P, d, args.steps, elapsed_ms / 1e3)
 
-    # roofline of the dominant kernel: fused accumulate + insert (20 algorithmic HBM bytes per
-    # worker-coordinate: read g, u, e; write u, e)
-    # per worker-coordinate, plus 4 bytes (re-read e) for every extra row pass
+    # Roofline of the dominant phase, the insert: per worker-coordinate 20 algorithmic HBM
+    # bytes for the fused accumulate + insert (read g, u, e; write u, e) plus 4 (re-read e)
+    # per extra row pass; for the sketched state, 4 bytes (read g) per row pass.  One launch
+    # of the kernel covers one group of W workers, so a phase is `groups` x `passes` launches.
     peaks, peak_kind = measured_peaks()
     rpp = gs.gs_sketch_info(sk)["rows_per_pass"]
     passes = -(-r // rpp)
-    per_wc = 20.0 + 4.0 * (passes - 1)
-    k1_bytes = [per_wc * n * d for n in k1_lanes]
-    k1_avg_s = (sum(k1_ms) / len(k1_ms)) / 1e3
-    k1_gbs = (sum(k1_bytes) / len(k1_bytes)) / k1_avg_s / 1e9
-    full_launch_bytes = per_wc * W * d
-    reds_per_launch = d * r * ((W + 3) // 4)
-    if variant == "sketched_state":
-        # the timed unit is the whole composed call: read g once per row pass (4 B per
-        # worker-coordinate and pass), write and re-read the estimate (8 B per coordinate)
-        per_wc = 4.0 * passes
-        full_launch_bytes = per_wc * P * d + 8.0 * d
-        k1_gbs = full_launch_bytes / k1_avg_s / 1e9
+    per_wc = 4.0 * passes if variant == "sketched_state" else 20.0 + 4.0 * (passes - 1)
+    phase_s = (sum(k1_ms) / len(k1_ms)) / 1e3
+    phase_bytes = per_wc * P * d
+    k1_gbs = phase_bytes / phase_s / 1e9
+    cells = d * r * groups
     roofline = {
-        "kernel": "gs_sketched_state_step (whole composed call)" if variant == "sketched_state" else
-                  "k_accumulate_insert (fused S1+S2), one call = one group of workers, all row passes",
-        "row_passes": passes, "algorithmic_bytes_per_worker_coord": per_wc,
+        "kernel": ("k_accumulate_insert_coop (insert only" if variant == "sketched_state" else
+                   "k_accumulate_insert_coop (fused S1+S2") + f", W={W}), the insert phase of a step: "
+                  f"{groups} group(s) x {passes} row pass(es)",
+        "row_passes": passes, "groups": groups, "algorithmic_bytes_per_worker_coord": per_wc,
         "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
         "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
-        "traffic": k1_traffic_per_launch() if variant != "sketched_state" else None,
-        "algorithmic_bytes_per_launch": full_launch_bytes,
-        "avg_launch_ms": round(sum(k1_ms) / len(k1_ms), 4),
-        "co_bound": {"kind": "l2_reductions, 16-byte requests merged per 32-byte cell",
-                     "cell_updates_per_launch": d * r * (groups if variant == "sketched_state" else 1),
-                     "achieved_G_cells_per_s": round(d * r * (groups if variant == "sketched_state" else 1)
-                                                     / k1_avg_s / 1e9, 1),
+        "traffic": k1_traffic_per_launch() if variant != "sketched_state" and groups * passes == 1 else None,
+        "algorithmic_bytes_per_launch": phase_bytes / (groups * passes) if passes == 1 else None,
+        "algorithmic_bytes_per_phase": phase_bytes,
+        "avg_launch_ms": round(sum(k1_ms) / len(k1_ms) / (groups * passes), 4),
+        "avg_phase_ms": round(sum(k1_ms) / len(k1_ms), 4),
+        "timed_phases": len(k1_ms),
+        "timing": "event-record nodes inside the step's CUDA graph" if use_plan else "CUDA events around the call",
+        "co_bound": {"kind": "l2_reductions, one 32-byte request per cell update (W=8)",
+                     "cell_updates_per_phase": cells,
+                     "achieved_G_cells_per_s": round(cells / phase_s / 1e9, 1),
                      "probe_peak_G_cells_per_s": 134.5},
         "step_share": round(sum(k1_ms) / elapsed_ms, 3),
     }
 
-    # end to end through the public call with host buffers
+    # end to end through the public API with host buffers: a host plan per gradient set (the
+    # uploads where needed, the step and the download of idx and vals are one graph), then a
+    # stream synchronisation so that the host can read the step's result
     e2e = None
     if not args.no_e2e and not args.profile_steps and variant == "error_feedback":
         grad_dev = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(P)]
         idx_h = torch.empty(k, dtype=torch.int64).pin_memory()
         vals_h = torch.empty(k, dtype=torch.float32).pin_memory()
+        hplans = []
+        if use_plan:
+            hplans = [gs.gs_step_host_plan_create(sk, us, es, hb, grad_dev, d, rho, k, idx_h, vals_h, ws)
+                      for hb in host_pool]
+
+        def host_step(t):
+            if use_plan:
+                gs.gs_plan_launch(hplans[t % len(hplans)], stream)
+                stream.synchronize()
+            else:
+                gs.gs_step_host(sk, us, es, host_pool[t % len(host_pool)], grad_dev, d, rho, k, idx_h, vals_h, ws,
+                                None, stream)
+
         for t in range(args.warmup):
-            gs.gs_step_host(sk, us, es, host_pool[t % len(host_pool)], grad_dev, d, rho, k, idx_h, vals_h, ws,
-                            None, stream)
+            host_step(t)
         if world > 1:
             import torch.distributed as dist
             dist.barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         for t in range(args.steps):
-            gs.gs_step_host(sk, us, es, host_pool[(args.warmup + t) % len(host_pool)], grad_dev, d, rho, k, idx_h,
-                            vals_h, ws, None, stream)
+            host_step(args.warmup + t)
         torch.cuda.synchronize()
         e2e_s = time.perf_counter() - t0
         if world > 1:
             import torch.distributed as dist
             dist.barrier()
         e2e_s = dist_max(e2e_s, dev)
+        for hp in hplans:
+            gs.gs_plan_destroy(hp)
         e2e = {"value": whole_job_rate(world, P, d, args.steps, e2e_s), "unit": UNIT, "h2d_bytes_per_step": P * d * 4,
                "d2h_bytes_per_step": k * (8 + 4), "ms_per_step": round(e2e_s * 1e3 / args.steps, 4),
-               "call": "gs_step_host"}
+               "call": "gs_step_host_plan_create + gs_plan_launch" if use_plan else "gs_step_host"}
+
+    for plan in plans:
+        gs.gs_plan_destroy(plan)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_steps \
@@ -405,7 +436,7 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": w.name, "variant": variant, "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
+        "config": {"workload": w.name, "variant": variant, "launch": "plan" if use_plan else "eager", "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
                    "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
                    "l2": f"inputs larger than L2 ({P * d * 12 / 1e9:.2f} GB of g,u,e streamed per step)",
                    "d_steps_per_s": world * d * args.steps / (elapsed_ms / 1e3)},

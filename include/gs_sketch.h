@@ -57,6 +57,7 @@ typedef int32_t gs_status;
 
 typedef struct gs_sketch gs_sketch; /* opaque */
 typedef void* gs_stream;            /* a cudaStream_t */
+typedef struct gs_plan gs_plan;     /* opaque: one step captured into a CUDA graph */
 
 /* ---- sketch lifetime ------------------------------------------------------------- */
 
@@ -283,6 +284,61 @@ gs_status gs_step_host(gs_sketch* sketch, float* const* momentum, float* const* 
                        const float* const* grad_host, float* const* grad_dev, int64_t d,
                        float rho, int64_t k, int64_t* idx_host, float* vals_host,
                        void* workspace, size_t workspace_bytes, gs_stream stream);
+
+/* ---- plans: a whole step captured once, launched many times ----------------------- */
+/* A plan records one step's launch sequence (the same kernels, order and arguments as the
+ * matching call above) into a CUDA graph, so that each later step is a single graph launch
+ * instead of one launch per kernel and memset.  It has no counterpart in the paper: it only
+ * removes host launch overhead and the gaps between dependent launches.
+ *
+ * A plan holds the POINTERS it was created with, not the data behind them: refill the
+ * gradients in place between launches; momentum, error, sketch tables, workspace and outputs
+ * are reused as in the direct calls.  All of them must stay allocated until
+ * gs_plan_destroy.  The sketches must not be destroyed first.  A plan is not thread-safe.
+ *
+ * flags: 0, or GS_PLAN_TIME_INSERT to bracket the insert phase (zeroed tables excluded) with
+ * two event-record nodes; launch n records into slot n mod 1024 of a ring of event pairs, and
+ * gs_plan_insert_times reads them.
+ *
+ * Errors: the same argument checks as the direct call (GS_ERR_INVALID_ARG, GS_ERR_MISMATCH);
+ * GS_ERR_CUDA if capture or instantiation fails (for example a host gradient that is neither
+ * device-addressable nor pinned, whose upload cannot be captured).  Nothing is launched while
+ * a plan is created. */
+#define GS_PLAN_TIME_INSERT 1
+
+/* gs_step (weights == NULL) or gs_train_step (weights != NULL, with lr) as a plan. */
+gs_status gs_step_plan_create(gs_sketch* sketch, float* const* momentum, float* const* error,
+                              const float* const* grad, int64_t d, float rho, int64_t k,
+                              int64_t* idx_out, float* vals_out, float* est_out, float* weights,
+                              float lr, void* workspace, size_t workspace_bytes, int32_t flags,
+                              gs_plan** plan_out);
+
+/* gs_step_host as a plan.  The uploads (where needed) and the download of idx and vals into
+ * idx_host / vals_host are part of the graph; a launch does NOT synchronise: synchronise the
+ * stream before reading the host outputs. */
+gs_status gs_step_host_plan_create(gs_sketch* sketch, float* const* momentum, float* const* error,
+                                   const float* const* grad_host, float* const* grad_dev,
+                                   int64_t d, float rho, int64_t k, int64_t* idx_host,
+                                   float* vals_host, void* workspace, size_t workspace_bytes,
+                                   int32_t flags, gs_plan** plan_out);
+
+/* gs_sketched_state_step as a plan. */
+gs_status gs_sketched_state_plan_create(gs_sketch* workers, gs_sketch* momentum, gs_sketch* error,
+                                        const float* const* grad, int64_t d, float rho, int64_t k,
+                                        int64_t* idx_out, float* vals_out, float* weights, float lr,
+                                        void* workspace, size_t workspace_bytes, int32_t flags,
+                                        gs_plan** plan_out);
+
+/* Enqueue one step on `stream` (asynchronous). */
+gs_status gs_plan_launch(gs_plan* plan, gs_stream stream);
+
+/* Insert-phase durations in ms of the last min(n, launches, 1024) launches, oldest first,
+ * into ms_out (host); *n_out = how many.  Waits for the last launch to finish.
+ * GS_ERR_INVALID_ARG if the plan was created without GS_PLAN_TIME_INSERT. */
+gs_status gs_plan_insert_times(gs_plan* plan, float* ms_out, int32_t n, int32_t* n_out);
+
+/* Wait for the device to go idle if the plan was ever launched, then free it.  NULL is OK. */
+gs_status gs_plan_destroy(gs_plan* plan);
 
 /* ---- inspection hooks ------------------------------------------------------------ */
 

@@ -57,6 +57,15 @@ SIGNATURES = {
     "gs_sketch_query_at": [_vp, _vp, _i64, _vp, _vp],
     "gs_sketch_add_sparse": [_vp, _vp, _vp, _i64, _f32, _vp],
     "gs_sketched_state_step": [_vp, _vp, _vp, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _f32, _vp, _sz, _vp],
+    "gs_step_plan_create": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _f32, _vp, _sz, _i32,
+                            ctypes.POINTER(_vp)],
+    "gs_step_host_plan_create": [_vp, _PP, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _sz, _i32,
+                                 ctypes.POINTER(_vp)],
+    "gs_sketched_state_plan_create": [_vp, _vp, _vp, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _f32, _vp, _sz, _i32,
+                                      ctypes.POINTER(_vp)],
+    "gs_plan_launch": [_vp, _vp],
+    "gs_plan_insert_times": [_vp, _vp, _i32, ctypes.POINTER(_i32)],
+    "gs_plan_destroy": [_vp],
     "gs_step_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_step": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
     "gs_step_host": [_vp, _PP, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _sz, _vp],
@@ -283,6 +292,62 @@ def gs_step_host(sketch: int, momentum, error, grad_host, grad_dev, d: int, rho:
     _check(load_library().gs_step_host(sketch, _ptr_array(momentum), _ptr_array(error), _ptr_array(grad_host),
                                        _ptr_array(grad_dev), d, rho, k, _ptr(idx_host), _ptr(vals_host),
                                        _ptr(workspace), workspace_bytes, _stream(stream)), "gs_step_host")
+
+
+GS_PLAN_TIME_INSERT = 1
+
+
+def _nbytes(workspace, workspace_bytes):
+    return workspace.numel() * workspace.element_size() if workspace_bytes is None else workspace_bytes
+
+
+def gs_step_plan_create(sketch: int, momentum, error, grad, d: int, rho: float, k: int, idx_out, vals_out,
+                        est_out=None, weights=None, lr: float = 0.0, workspace=None, workspace_bytes=None,
+                        flags: int = 0) -> int:
+    out = _vp()
+    _check(load_library().gs_step_plan_create(sketch, _ptr_array(momentum), _ptr_array(error), _ptr_array(grad), d,
+                                              rho, k, _ptr(idx_out), _ptr(vals_out), _ptr(est_out), _ptr(weights), lr,
+                                              _ptr(workspace), _nbytes(workspace, workspace_bytes), flags,
+                                              ctypes.byref(out)), "gs_step_plan_create")
+    return out.value
+
+
+def gs_step_host_plan_create(sketch: int, momentum, error, grad_host, grad_dev, d: int, rho: float, k: int,
+                             idx_host, vals_host, workspace, workspace_bytes=None, flags: int = 0) -> int:
+    out = _vp()
+    _check(load_library().gs_step_host_plan_create(sketch, _ptr_array(momentum), _ptr_array(error),
+                                                   _ptr_array(grad_host), _ptr_array(grad_dev), d, rho, k,
+                                                   _ptr(idx_host), _ptr(vals_host), _ptr(workspace),
+                                                   _nbytes(workspace, workspace_bytes), flags, ctypes.byref(out)),
+           "gs_step_host_plan_create")
+    return out.value
+
+
+def gs_sketched_state_plan_create(workers: int, momentum: int, error: int, grad, d: int, rho: float, k: int,
+                                  idx_out, vals_out, weights, lr: float, workspace, workspace_bytes=None,
+                                  flags: int = 0) -> int:
+    out = _vp()
+    _check(load_library().gs_sketched_state_plan_create(workers, momentum, error, _ptr_array(grad), d, rho, k,
+                                                        _ptr(idx_out), _ptr(vals_out), _ptr(weights), lr,
+                                                        _ptr(workspace), _nbytes(workspace, workspace_bytes), flags,
+                                                        ctypes.byref(out)), "gs_sketched_state_plan_create")
+    return out.value
+
+
+def gs_plan_launch(plan: int, stream=None) -> None:
+    _check(load_library().gs_plan_launch(plan, _stream(stream)), "gs_plan_launch")
+
+
+def gs_plan_insert_times(plan: int, n: int = 1024) -> list:
+    buf = (ctypes.c_float * max(n, 1))()
+    got = _i32()
+    _check(load_library().gs_plan_insert_times(plan, ctypes.cast(buf, _vp), n, ctypes.byref(got)),
+           "gs_plan_insert_times")
+    return [float(buf[i]) for i in range(got.value)]
+
+
+def gs_plan_destroy(plan: int) -> None:
+    _check(load_library().gs_plan_destroy(plan), "gs_plan_destroy")
 
 
 def gs_hash_eval(sketch: int, coords, n: int, bucket_out, sign_out, stream=None) -> None:

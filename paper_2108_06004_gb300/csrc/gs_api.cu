@@ -19,6 +19,16 @@ struct gs_sketch {
   int device;
 };
 
+struct gs_plan {
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  bool timed = false;
+  cudaGraphNode_t node_begin = nullptr, node_end = nullptr;  // event-record nodes around the insert phase
+  std::vector<cudaEvent_t> ev_begin, ev_end;                 // their ring of events
+  int64_t launches = 0;
+  int device = 0;
+};
+
 namespace {
 
 thread_local std::string g_err;
@@ -196,14 +206,27 @@ bool same_family(const gs_sketch* a, const gs_sketch* b) {
   return a->r == b->r && a->c == b->c && a->seed == b->seed;
 }
 
+// Optional events recorded around the insert phase of a step.  They are used only while a
+// step is captured into a plan, where each becomes an event-record node of the graph.
+struct InsertMarks {
+  cudaEvent_t begin = nullptr, end = nullptr;
+};
+
+cudaError_t mark(cudaEvent_t ev, cudaStream_t s) {
+  return ev ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal) : cudaSuccess;
+}
+
 gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float* const* g,
                     int64_t d, float rho, int64_t k, int64_t* idx, float* vals, float* est,
-                    void* ws, cudaStream_t s, float* weights = nullptr, float lr = 0.f) {
+                    void* ws, cudaStream_t s, float* weights = nullptr, float lr = 0.f,
+                    InsertMarks marks = InsertMarks()) {
   const size_t bytes = (size_t)sk->groups * sk->r * sk->c * sk->W * sizeof(float) +
                        (size_t)sk->r * sk->c * sizeof(float);
   cudaError_t err = cudaMemsetAsync(sk->tables, 0, bytes, s);
   if (err != cudaSuccess) return cuda_fail(err, "zero tables");
+  if ((err = mark(marks.begin, s)) != cudaSuccess) return cuda_fail(err, "event record");
   GS_TRY(accumulate_insert_impl(sk, 0, sk->workers, m, e, g, d, rho, s));
+  if ((err = mark(marks.end, s)) != cudaSuccess) return cuda_fail(err, "event record");
   gs::MergeParams mp;
   mp.tables = sk->tables;
   mp.merged = sk->merged;
@@ -244,6 +267,252 @@ gs_status check_worker_arrays(int n, float* const* m, float* const* e, const flo
 size_t step_ws_bytes(int64_t d, int64_t k) {
   return gs::query_topk_workspace_bytes(d, k) + (((size_t)k * 8 + 255) & ~size_t(255)) +
          (((size_t)k * 4 + 255) & ~size_t(255));
+}
+
+gs_status check_sketched_state(gs_sketch* workers, gs_sketch* momentum, gs_sketch* error, const float* const* grad,
+                               int64_t d, int64_t k, int64_t* idx_out, float* vals_out, float* weights,
+                               void* workspace, size_t workspace_bytes) {
+  GS_TRY(check_sketch(workers));
+  GS_TRY(check_sketch(momentum));
+  GS_TRY(check_sketch(error));
+  if (!same_family(workers, momentum) || !same_family(workers, error))
+    return fail(GS_ERR_MISMATCH, "the three sketches must share r, c and seed");
+  if (momentum == error || momentum == workers || error == workers)
+    return fail(GS_ERR_INVALID_ARG, "workers, momentum and error must be three different sketches");
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  for (int p = 0; p < workers->workers; ++p) GS_TRY(check_vec(grad[p], "grad[p]"));
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals_out, "vals_out"));
+  if (weights) GS_TRY(check_vec(weights, "weights"));
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < step_ws_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_step_workspace_size");
+  return GS_OK;
+}
+
+// S = tree merge of S(g_p); U <- rho U + S, E <- E + U; top-k of the estimate from E; the
+// extracted mass leaves E and U.  Arguments already checked.
+gs_status sketched_state_impl(gs_sketch* workers, gs_sketch* momentum, gs_sketch* error, const float* const* grad,
+                              int64_t d, float rho, int64_t k, int64_t* idx, float* vals, float* weights, float lr,
+                              void* ws, cudaStream_t s, InsertMarks marks = InsertMarks()) {
+  const int64_t cells = (int64_t)workers->r * workers->c;
+  // S = tree merge of S(g_p)
+  const size_t tbytes = ((size_t)workers->groups * workers->r * workers->c * workers->W + (size_t)cells) * sizeof(float);
+  cudaError_t err = cudaMemsetAsync(workers->tables, 0, tbytes, s);
+  if (err != cudaSuccess) return cuda_fail(err, "zero tables");
+  if ((err = mark(marks.begin, s)) != cudaSuccess) return cuda_fail(err, "event record");
+  GS_TRY(insert_all_impl(workers, grad, d, s));
+  if ((err = mark(marks.end, s)) != cudaSuccess) return cuda_fail(err, "event record");
+  gs::MergeParams mp;
+  mp.tables = workers->tables;
+  mp.merged = workers->merged;
+  mp.cells = cells;
+  mp.group_stride = cells * workers->W;
+  mp.P = workers->workers;
+  if ((err = gs::launch_merge(mp, workers->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
+  // U <- rho U + S ; E <- E + U   (elementwise on the r*c cells)
+  if ((err = gs::launch_accumulate(momentum->merged, error->merged, workers->merged, cells, rho, s)) != cudaSuccess)
+    return cuda_fail(err, "sketch accumulate launch");
+  // top-k of the estimate from E; delta = that estimate at the selected coordinates
+  if ((err = gs::launch_query_topk(error->merged, error->h, error->r, (uint32_t)error->c, d, k, idx, nullptr,
+                                   ws, s)) != cudaSuccess)
+    return cuda_fail(err, "query/top-k launch");
+  const float* est = static_cast<const float*>(ws);  // the query keeps est at the ws start
+  if ((err = gs::launch_take(est, d, idx, k, vals, s)) != cudaSuccess) return cuda_fail(err, "take launch");
+  float* delta_u = reinterpret_cast<float*>(static_cast<char*>(ws) + gs::query_topk_workspace_bytes(d, k));
+  if ((err = gs::launch_query_at(momentum->merged, momentum->h, momentum->r, (uint32_t)momentum->c, idx, k,
+                                 delta_u, s)) != cudaSuccess)
+    return cuda_fail(err, "query_at launch");
+  // the extracted mass leaves both sketches
+  if ((err = gs::launch_add_sparse(error->merged, error->h, error->r, (uint32_t)error->c, idx, vals, k, -1.f,
+                                   s)) != cudaSuccess)
+    return cuda_fail(err, "add_sparse launch");
+  if ((err = gs::launch_add_sparse(momentum->merged, momentum->h, momentum->r, (uint32_t)momentum->c, idx, delta_u,
+                                   k, -1.f, s)) != cudaSuccess)
+    return cuda_fail(err, "add_sparse launch");
+  if (weights && (err = gs::launch_apply_update(weights, d, idx, vals, k, lr, s)) != cudaSuccess)
+    return cuda_fail(err, "update launch");
+  return GS_OK;
+}
+
+gs_status check_step(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad, int64_t d,
+                     int64_t k, int64_t* idx_out, float* vals_out, float* est_out, void* workspace,
+                     size_t workspace_bytes) {
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad));
+  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
+  GS_TRY(check_vec(vals_out, "vals_out"));
+  if (est_out) GS_TRY(check_vec(est_out, "est_out"));
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < gs::query_topk_workspace_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small");
+  return GS_OK;
+}
+
+gs_status check_host_step(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad_host,
+                          float* const* grad_dev, int64_t d, int64_t k, int64_t* idx_host, float* vals_host,
+                          void* workspace, size_t workspace_bytes) {
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!grad_host || !grad_dev) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  for (int p = 0; p < sk->workers; ++p)
+    if (!grad_host[p]) return fail(GS_ERR_INVALID_ARG, "grad_host[p] is NULL");
+  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad_dev));
+  if (!idx_host || !vals_host) return fail(GS_ERR_INVALID_ARG, "host outputs are NULL");
+  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < step_ws_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_step_workspace_size");
+  return GS_OK;
+}
+
+// Where the fused kernel reads each worker's host gradient: the gradient itself where the GPU
+// can address it (pinned or registered host memory, device memory, or any host memory when
+// the device has pageable-memory access), else nullptr: first copied into grad_dev[p].
+void host_sources(const gs_sketch* sk, const float* const* grad_host, float* const* grad_dev,
+                  std::vector<const float*>& src) {
+  int pageable = 0;
+  cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, sk->device);
+  src.assign((size_t)sk->workers, nullptr);
+  for (int p = 0; p < sk->workers; ++p) {
+    cudaPointerAttributes attr;
+    if (cudaPointerGetAttributes(&attr, grad_host[p]) != cudaSuccess) {
+      cudaGetLastError();
+      attr.type = cudaMemoryTypeUnregistered;
+      attr.devicePointer = nullptr;
+    }
+    const float* direct = nullptr;
+    if (attr.type == cudaMemoryTypeHost && attr.devicePointer) direct = static_cast<const float*>(attr.devicePointer);
+    else if (attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged) direct = grad_host[p];
+    else if (attr.type == cudaMemoryTypeUnregistered && pageable == 1) direct = grad_host[p];
+    if (direct && aligned(direct, 4)) src[(size_t)p] = direct;
+  }
+}
+
+// The host step on stream s: uploads where needed, the whole step, and the download of the
+// k indices and values into the host outputs (not synchronised).
+gs_status host_step_enqueue(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad_host,
+                            float* const* grad_dev, const std::vector<const float*>& src, int64_t d, float rho,
+                            int64_t k, int64_t* idx_host, float* vals_host, void* workspace, cudaStream_t s,
+                            InsertMarks marks = InsertMarks()) {
+  const size_t qbytes = gs::query_topk_workspace_bytes(d, k);
+  int64_t* idx_dev = reinterpret_cast<int64_t*>(static_cast<char*>(workspace) + qbytes);
+  float* vals_dev = reinterpret_cast<float*>(reinterpret_cast<char*>(idx_dev) + (((size_t)k * 8 + 255) & ~size_t(255)));
+  std::vector<const float*> gsrc(src);
+  for (int p = 0; p < sk->workers; ++p) {
+    if (gsrc[(size_t)p]) continue;
+    cudaError_t e = cudaMemcpyAsync(grad_dev[p], grad_host[p], (size_t)d * sizeof(float), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
+    gsrc[(size_t)p] = grad_dev[p];
+  }
+  GS_TRY(step_impl(sk, momentum, error, gsrc.data(), d, rho, k, idx_dev, vals_dev, nullptr, workspace, s, nullptr, 0.f,
+                   marks));
+  cudaError_t e = cudaMemcpyAsync(idx_host, idx_dev, (size_t)k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(vals_host, vals_dev, (size_t)k * sizeof(float), cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return cuda_fail(e, "result download");
+  return GS_OK;
+}
+
+// A plan's events for the insert phase are a ring: launch n records into slot n mod kPlanRing.
+constexpr int64_t kPlanRing = 1024;
+
+void plan_free(gs_plan* p) {
+  if (p->exec) cudaGraphExecDestroy(p->exec);
+  if (p->graph) cudaGraphDestroy(p->graph);
+  for (cudaEvent_t ev : p->ev_begin)
+    if (ev) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : p->ev_end)
+    if (ev) cudaEventDestroy(ev);
+  delete p;
+}
+
+gs_status check_plan(const gs_plan* plan) {
+  if (!plan) return fail(GS_ERR_INVALID_ARG, "plan is NULL");
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev != plan->device) return fail(GS_ERR_INVALID_ARG, "current device differs from the plan's device");
+  return GS_OK;
+}
+
+// Capture body(stream, marks) on a private stream into a graph and instantiate it.  With
+// GS_PLAN_TIME_INSERT the insert phase is bracketed by two event-record nodes whose events
+// each launch re-points into the ring.
+template <class Body>
+gs_status capture_plan(int device, int32_t flags, gs_plan** out, Body&& body) {
+  if (!out) return fail(GS_ERR_INVALID_ARG, "plan_out is NULL");
+  if (flags & ~int32_t(GS_PLAN_TIME_INSERT)) return fail(GS_ERR_INVALID_ARG, "unknown plan flags");
+  gs_plan* p = new gs_plan();
+  p->device = device;
+  p->timed = (flags & GS_PLAN_TIME_INSERT) != 0;
+  cudaError_t e = cudaSuccess;
+  if (p->timed) {
+    p->ev_begin.assign((size_t)kPlanRing, nullptr);
+    p->ev_end.assign((size_t)kPlanRing, nullptr);
+    for (size_t i = 0; i < (size_t)kPlanRing && e == cudaSuccess; ++i) {
+      e = cudaEventCreate(&p->ev_begin[i]);
+      if (e == cudaSuccess) e = cudaEventCreate(&p->ev_end[i]);
+    }
+    if (e != cudaSuccess) {
+      plan_free(p);
+      return cuda_fail(e, "cudaEventCreate");
+    }
+  }
+  cudaStream_t cs = nullptr;
+  if ((e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking)) != cudaSuccess) {
+    plan_free(p);
+    return cuda_fail(e, "cudaStreamCreateWithFlags");
+  }
+  if ((e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal)) != cudaSuccess) {
+    cudaStreamDestroy(cs);
+    plan_free(p);
+    return cuda_fail(e, "cudaStreamBeginCapture");
+  }
+  InsertMarks marks;
+  if (p->timed) {
+    marks.begin = p->ev_begin[0];
+    marks.end = p->ev_end[0];
+  }
+  const gs_status st = body(cs, marks);
+  cudaGraph_t graph = nullptr;
+  e = cudaStreamEndCapture(cs, &graph);
+  cudaStreamDestroy(cs);
+  p->graph = graph;
+  if (st != GS_OK) {
+    plan_free(p);
+    return st;
+  }
+  if (e != cudaSuccess) {
+    plan_free(p);
+    return cuda_fail(e, "stream capture");
+  }
+  if (p->timed) {
+    size_t n = 0;
+    e = cudaGraphGetNodes(graph, nullptr, &n);
+    std::vector<cudaGraphNode_t> nodes(n);
+    if (e == cudaSuccess && n) e = cudaGraphGetNodes(graph, nodes.data(), &n);
+    for (size_t i = 0; i < n && e == cudaSuccess; ++i) {
+      cudaGraphNodeType type;
+      if ((e = cudaGraphNodeGetType(nodes[i], &type)) != cudaSuccess || type != cudaGraphNodeTypeEventRecord) continue;
+      cudaEvent_t ev = nullptr;
+      if ((e = cudaGraphEventRecordNodeGetEvent(nodes[i], &ev)) != cudaSuccess) break;
+      if (ev == marks.begin) p->node_begin = nodes[i];
+      if (ev == marks.end) p->node_end = nodes[i];
+    }
+    if (e == cudaSuccess && (!p->node_begin || !p->node_end)) {
+      plan_free(p);
+      return fail(GS_ERR_CUDA, "stream capture: insert-phase event nodes not found");
+    }
+  }
+  if (e == cudaSuccess) e = cudaGraphInstantiate(&p->exec, graph, 0);
+  if (e != cudaSuccess) {
+    plan_free(p);
+    return cuda_fail(e, "graph instantiation");
+  }
+  *out = p;
+  return GS_OK;
 }
 
 }  // namespace
@@ -589,16 +858,7 @@ gs_status gs_step(gs_sketch* sk, float* const* momentum, float* const* error, co
                   float rho, int64_t k, int64_t* idx_out, float* vals_out, float* est_out, void* workspace,
                   size_t workspace_bytes, gs_stream stream) {
   GS_GUARD_BEGIN
-  GS_TRY(check_sketch(sk));
-  GS_TRY(check_d(d));
-  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
-  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
-  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad));
-  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
-  GS_TRY(check_vec(vals_out, "vals_out"));
-  if (est_out) GS_TRY(check_vec(est_out, "est_out"));
-  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
-  if (workspace_bytes < gs::query_topk_workspace_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small");
+  GS_TRY(check_step(sk, momentum, error, grad, d, k, idx_out, vals_out, est_out, workspace, workspace_bytes));
   return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, est_out, workspace, as_stream(stream));
   GS_GUARD_END
 }
@@ -607,17 +867,8 @@ gs_status gs_train_step(gs_sketch* sk, float* weights, float lr, float* const* m
                         const float* const* grad, int64_t d, float rho, int64_t k, int64_t* idx_out, float* vals_out,
                         float* est_out, void* workspace, size_t workspace_bytes, gs_stream stream) {
   GS_GUARD_BEGIN
-  GS_TRY(check_sketch(sk));
-  GS_TRY(check_d(d));
   GS_TRY(check_vec(weights, "weights"));
-  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
-  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
-  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad));
-  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
-  GS_TRY(check_vec(vals_out, "vals_out"));
-  if (est_out) GS_TRY(check_vec(est_out, "est_out"));
-  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
-  if (workspace_bytes < gs::query_topk_workspace_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small");
+  GS_TRY(check_step(sk, momentum, error, grad, d, k, idx_out, vals_out, est_out, workspace, workspace_bytes));
   return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, est_out, workspace, as_stream(stream),
                    weights, lr);
   GS_GUARD_END
@@ -656,59 +907,10 @@ gs_status gs_sketched_state_step(gs_sketch* workers, gs_sketch* momentum, gs_ske
                                  int64_t d, float rho, int64_t k, int64_t* idx_out, float* vals_out, float* weights,
                                  float lr, void* workspace, size_t workspace_bytes, gs_stream stream) {
   GS_GUARD_BEGIN
-  GS_TRY(check_sketch(workers));
-  GS_TRY(check_sketch(momentum));
-  GS_TRY(check_sketch(error));
-  if (!same_family(workers, momentum) || !same_family(workers, error))
-    return fail(GS_ERR_MISMATCH, "the three sketches must share r, c and seed");
-  if (momentum == error || momentum == workers || error == workers)
-    return fail(GS_ERR_INVALID_ARG, "workers, momentum and error must be three different sketches");
-  GS_TRY(check_d(d));
-  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
-  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
-  for (int p = 0; p < workers->workers; ++p) GS_TRY(check_vec(grad[p], "grad[p]"));
-  if (!idx_out || !aligned(idx_out, 8)) return fail(GS_ERR_INVALID_ARG, "idx_out is NULL or not 8-byte aligned");
-  GS_TRY(check_vec(vals_out, "vals_out"));
-  if (weights) GS_TRY(check_vec(weights, "weights"));
-  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
-  if (workspace_bytes < step_ws_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_step_workspace_size");
-  cudaStream_t s = as_stream(stream);
-  const int64_t cells = (int64_t)workers->r * workers->c;
-  // S = tree merge of S(g_p)
-  const size_t tbytes = ((size_t)workers->groups * workers->r * workers->c * workers->W + (size_t)cells) * sizeof(float);
-  cudaError_t err = cudaMemsetAsync(workers->tables, 0, tbytes, s);
-  if (err != cudaSuccess) return cuda_fail(err, "zero tables");
-  GS_TRY(insert_all_impl(workers, grad, d, s));
-  gs::MergeParams mp;
-  mp.tables = workers->tables;
-  mp.merged = workers->merged;
-  mp.cells = cells;
-  mp.group_stride = cells * workers->W;
-  mp.P = workers->workers;
-  if ((err = gs::launch_merge(mp, workers->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
-  // U <- rho U + S ; E <- E + U   (elementwise on the r*c cells)
-  if ((err = gs::launch_accumulate(momentum->merged, error->merged, workers->merged, cells, rho, s)) != cudaSuccess)
-    return cuda_fail(err, "sketch accumulate launch");
-  // top-k of the estimate from E; delta = that estimate at the selected coordinates
-  if ((err = gs::launch_query_topk(error->merged, error->h, error->r, (uint32_t)error->c, d, k, idx_out, nullptr,
-                                   workspace, s)) != cudaSuccess)
-    return cuda_fail(err, "query/top-k launch");
-  const float* est = static_cast<const float*>(workspace);  // the query keeps est at the workspace start
-  if ((err = gs::launch_take(est, d, idx_out, k, vals_out, s)) != cudaSuccess) return cuda_fail(err, "take launch");
-  float* delta_u = reinterpret_cast<float*>(static_cast<char*>(workspace) + gs::query_topk_workspace_bytes(d, k));
-  if ((err = gs::launch_query_at(momentum->merged, momentum->h, momentum->r, (uint32_t)momentum->c, idx_out, k,
-                                 delta_u, s)) != cudaSuccess)
-    return cuda_fail(err, "query_at launch");
-  // the extracted mass leaves both sketches
-  if ((err = gs::launch_add_sparse(error->merged, error->h, error->r, (uint32_t)error->c, idx_out, vals_out, k, -1.f,
-                                   s)) != cudaSuccess)
-    return cuda_fail(err, "add_sparse launch");
-  if ((err = gs::launch_add_sparse(momentum->merged, momentum->h, momentum->r, (uint32_t)momentum->c, idx_out, delta_u,
-                                   k, -1.f, s)) != cudaSuccess)
-    return cuda_fail(err, "add_sparse launch");
-  if (weights && (err = gs::launch_apply_update(weights, d, idx_out, vals_out, k, lr, s)) != cudaSuccess)
-    return cuda_fail(err, "update launch");
-  return GS_OK;
+  GS_TRY(check_sketched_state(workers, momentum, error, grad, d, k, idx_out, vals_out, weights, workspace,
+                              workspace_bytes));
+  return sketched_state_impl(workers, momentum, error, grad, d, rho, k, idx_out, vals_out, weights, lr, workspace,
+                             as_stream(stream));
   GS_GUARD_END
 }
 
@@ -716,52 +918,108 @@ gs_status gs_step_host(gs_sketch* sk, float* const* momentum, float* const* erro
                        float* const* grad_dev, int64_t d, float rho, int64_t k, int64_t* idx_host, float* vals_host,
                        void* workspace, size_t workspace_bytes, gs_stream stream) {
   GS_GUARD_BEGIN
-  GS_TRY(check_sketch(sk));
-  GS_TRY(check_d(d));
-  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
-  if (!grad_host || !grad_dev) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
-  for (int p = 0; p < sk->workers; ++p)
-    if (!grad_host[p]) return fail(GS_ERR_INVALID_ARG, "grad_host[p] is NULL");
-  GS_TRY(check_worker_arrays(sk->workers, momentum, error, grad_dev));
-  if (!idx_host || !vals_host) return fail(GS_ERR_INVALID_ARG, "host outputs are NULL");
-  if (!workspace || !aligned(workspace, 256)) return fail(GS_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
-  if (workspace_bytes < step_ws_bytes(d, k)) return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_step_workspace_size");
+  GS_TRY(check_host_step(sk, momentum, error, grad_host, grad_dev, d, k, idx_host, vals_host, workspace,
+                         workspace_bytes));
+  std::vector<const float*> src;
+  host_sources(sk, grad_host, grad_dev, src);
   cudaStream_t s = as_stream(stream);
-  const size_t qbytes = gs::query_topk_workspace_bytes(d, k);
-  int64_t* idx_dev = reinterpret_cast<int64_t*>(static_cast<char*>(workspace) + qbytes);
-  float* vals_dev = reinterpret_cast<float*>(reinterpret_cast<char*>(idx_dev) + (((size_t)k * 8 + 255) & ~size_t(255)));
-  // Gradients the GPU can address in place (pinned or registered host memory, or any host
-  // memory where the device has pageable-memory access) are read by the fused kernel over
-  // the CPU-GPU link; others are first copied into grad_dev.
-  int pageable = 0;
-  cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, sk->device);
-  std::vector<const float*> gsrc((size_t)sk->workers);
-  for (int p = 0; p < sk->workers; ++p) {
-    cudaPointerAttributes attr;
-    cudaError_t e = cudaPointerGetAttributes(&attr, grad_host[p]);
-    if (e != cudaSuccess) {
-      cudaGetLastError();
-      attr.type = cudaMemoryTypeUnregistered;
-    }
-    const float* direct = nullptr;
-    if (attr.type == cudaMemoryTypeHost && attr.devicePointer) direct = static_cast<const float*>(attr.devicePointer);
-    else if (attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged) direct = grad_host[p];
-    else if (attr.type == cudaMemoryTypeUnregistered && pageable == 1) direct = grad_host[p];
-    if (direct && aligned(direct, 4)) {
-      gsrc[(size_t)p] = direct;
-    } else {
-      e = cudaMemcpyAsync(grad_dev[p], grad_host[p], (size_t)d * sizeof(float), cudaMemcpyHostToDevice, s);
-      if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
-      gsrc[(size_t)p] = grad_dev[p];
-    }
-  }
-  GS_TRY(step_impl(sk, momentum, error, gsrc.data(), d, rho, k, idx_dev, vals_dev, nullptr, workspace, s));
-  cudaError_t e = cudaMemcpyAsync(idx_host, idx_dev, (size_t)k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(vals_host, vals_dev, (size_t)k * sizeof(float), cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  GS_TRY(host_step_enqueue(sk, momentum, error, grad_host, grad_dev, src, d, rho, k, idx_host, vals_host, workspace, s));
+  cudaError_t e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "result download");
   return GS_OK;
   GS_GUARD_END
+}
+
+// ---- plans: one step captured into a CUDA graph -------------------------------------------
+
+gs_status gs_step_plan_create(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad,
+                              int64_t d, float rho, int64_t k, int64_t* idx_out, float* vals_out, float* est_out,
+                              float* weights, float lr, void* workspace, size_t workspace_bytes, int32_t flags,
+                              gs_plan** plan_out) {
+  GS_GUARD_BEGIN
+  if (plan_out) *plan_out = nullptr;
+  GS_TRY(check_step(sk, momentum, error, grad, d, k, idx_out, vals_out, est_out, workspace, workspace_bytes));
+  if (weights) GS_TRY(check_vec(weights, "weights"));
+  return capture_plan(sk->device, flags, plan_out, [&](cudaStream_t s, InsertMarks marks) {
+    return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, est_out, workspace, s, weights, lr,
+                     marks);
+  });
+  GS_GUARD_END
+}
+
+gs_status gs_step_host_plan_create(gs_sketch* sk, float* const* momentum, float* const* error,
+                                   const float* const* grad_host, float* const* grad_dev, int64_t d, float rho,
+                                   int64_t k, int64_t* idx_host, float* vals_host, void* workspace,
+                                   size_t workspace_bytes, int32_t flags, gs_plan** plan_out) {
+  GS_GUARD_BEGIN
+  if (plan_out) *plan_out = nullptr;
+  GS_TRY(check_host_step(sk, momentum, error, grad_host, grad_dev, d, k, idx_host, vals_host, workspace,
+                         workspace_bytes));
+  std::vector<const float*> src;
+  host_sources(sk, grad_host, grad_dev, src);
+  return capture_plan(sk->device, flags, plan_out, [&](cudaStream_t s, InsertMarks marks) {
+    return host_step_enqueue(sk, momentum, error, grad_host, grad_dev, src, d, rho, k, idx_host, vals_host, workspace,
+                             s, marks);
+  });
+  GS_GUARD_END
+}
+
+gs_status gs_sketched_state_plan_create(gs_sketch* workers, gs_sketch* momentum, gs_sketch* error,
+                                        const float* const* grad, int64_t d, float rho, int64_t k, int64_t* idx_out,
+                                        float* vals_out, float* weights, float lr, void* workspace,
+                                        size_t workspace_bytes, int32_t flags, gs_plan** plan_out) {
+  GS_GUARD_BEGIN
+  if (plan_out) *plan_out = nullptr;
+  GS_TRY(check_sketched_state(workers, momentum, error, grad, d, k, idx_out, vals_out, weights, workspace,
+                              workspace_bytes));
+  return capture_plan(workers->device, flags, plan_out, [&](cudaStream_t s, InsertMarks marks) {
+    return sketched_state_impl(workers, momentum, error, grad, d, rho, k, idx_out, vals_out, weights, lr, workspace, s,
+                               marks);
+  });
+  GS_GUARD_END
+}
+
+gs_status gs_plan_launch(gs_plan* plan, gs_stream stream) {
+  GS_TRY(check_plan(plan));
+  cudaError_t e = cudaSuccess;
+  if (plan->timed) {
+    const size_t slot = (size_t)(plan->launches % kPlanRing);
+    e = cudaGraphExecEventRecordNodeSetEvent(plan->exec, plan->node_begin, plan->ev_begin[slot]);
+    if (e == cudaSuccess) e = cudaGraphExecEventRecordNodeSetEvent(plan->exec, plan->node_end, plan->ev_end[slot]);
+    if (e != cudaSuccess) return cuda_fail(e, "plan event update");
+  }
+  e = cudaGraphLaunch(plan->exec, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGraphLaunch");
+  ++plan->launches;
+  return GS_OK;
+}
+
+gs_status gs_plan_insert_times(gs_plan* plan, float* ms_out, int32_t n, int32_t* n_out) {
+  GS_TRY(check_plan(plan));
+  if (!plan->timed) return fail(GS_ERR_INVALID_ARG, "the plan was created without GS_PLAN_TIME_INSERT");
+  if (!ms_out || !n_out || n < 0) return fail(GS_ERR_INVALID_ARG, "ms_out or n_out is NULL, or n < 0");
+  int64_t m = n;
+  if (m > plan->launches) m = plan->launches;
+  if (m > kPlanRing) m = kPlanRing;
+  *n_out = 0;
+  if (m == 0) return GS_OK;
+  cudaError_t e = cudaEventSynchronize(plan->ev_end[(size_t)((plan->launches - 1) % kPlanRing)]);
+  for (int64_t t = 0; t < m && e == cudaSuccess; ++t) {
+    const size_t slot = (size_t)((plan->launches - m + t) % kPlanRing);
+    e = cudaEventElapsedTime(&ms_out[t], plan->ev_begin[slot], plan->ev_end[slot]);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "plan event times");
+  *n_out = (int32_t)m;
+  return GS_OK;
+}
+
+gs_status gs_plan_destroy(gs_plan* plan) {
+  if (!plan) return GS_OK;
+  cudaError_t e = cudaSuccess;
+  if (plan->launches > 0) e = cudaDeviceSynchronize();
+  plan_free(plan);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  return GS_OK;
 }
 
 gs_status gs_hash_eval(const gs_sketch* sk, const int64_t* coords, int64_t n, int32_t* bucket_out, int8_t* sign_out,

@@ -74,6 +74,19 @@ def test_validation_before_device_work(lib):
     assert lib.gs_gather_and_zero(arr, arr, 0, 10, 64, 1, 128, None) == gs.GS_ERR_INVALID_ARG
     assert lib.gs_gather_and_zero(arr, arr, 65, 10, 64, 1, 128, None) == gs.GS_ERR_INVALID_ARG
     assert lib.gs_gather_and_zero(arr, arr, 2, 10, 64, 11, 128, None) == gs.GS_ERR_INVALID_ARG
+    # plans: argument errors before any capture
+    plan = ctypes.c_void_p(12345)
+    assert lib.gs_step_plan_create(None, arr, arr, arr, 10, 0.9, 1, 64, 128, None, None, 0.0, 256, 1 << 20, 0,
+                                   ctypes.byref(plan)) == gs.GS_ERR_INVALID_ARG
+    assert plan.value is None and b"sketch is NULL" in lib.gs_last_error()
+    assert lib.gs_sketched_state_plan_create(None, None, None, arr, 10, 0.9, 1, 64, 128, None, 0.0, 256, 1 << 20, 0,
+                                             ctypes.byref(plan)) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_step_host_plan_create(None, arr, arr, arr, arr, 10, 0.9, 1, 64, 128, 256, 1 << 20, 0,
+                                        ctypes.byref(plan)) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_plan_launch(None, None) == gs.GS_ERR_INVALID_ARG
+    n_out = ctypes.c_int32()
+    assert lib.gs_plan_insert_times(None, None, 1, ctypes.byref(n_out)) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_plan_destroy(None) == gs.GS_OK
 
 
 def test_binding_raises_on_error(lib):

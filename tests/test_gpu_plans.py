@@ -1,0 +1,195 @@
+"""Plans: a whole step captured into a CUDA graph and launched many times.
+
+A plan launch must give what the direct call gives: the same agreement with the oracle,
+step after step, with the gradients refilled in place between launches (the plan holds
+pointers, not data).  Also checked: the timed insert phase yields one positive duration per
+launch, the host-buffer plan returns its results to host memory after a stream
+synchronisation, and the sketched-state plan follows the oracle like the direct call.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def gs():
+    import paper_2108_06004_gb300 as lib
+    lib.load_library()
+    return lib
+
+
+@pytest.fixture(scope="module")
+def H(gs):
+    from tests import gpu_harness
+    return gpu_harness
+
+
+def _dev(x):
+    return torch.from_numpy(np.ascontiguousarray(x)).to("cuda")
+
+
+@pytest.mark.parametrize("P,d,r,c,k,W,train", [
+    (4, 100_003, 5, 8192, 300, 0, False),
+    (6, 65_537, 3, 4099, 50, 2, True),
+    (8, 1 << 20, 5, 1 << 14, 1000, 0, False),
+])
+def test_step_plan(gs, H, P, d, r, c, k, W, train):
+    w = workloads.get_config("resnet18")
+    seed, lr = 29 + P, 0.05
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho, group_width=W)
+    gbuf = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+    weights = _dev(np.random.default_rng(5).standard_normal(d).astype(np.float32)) if train else None
+    plan = gs.gs_step_plan_create(run.sketch, run.us, run.es, gbuf, d, w.rho, k, run.idx, run.vals, run.est,
+                                  weights, lr, run.ws, flags=gs.GS_PLAN_TIME_INSERT)
+    try:
+        steps = 3
+        for t in range(steps):
+            grads = workloads.make_gradients(w, t, range(P), d=d)
+            for b, g in zip(gbuf, grads):
+                b.copy_(torch.from_numpy(g))
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            w0 = H.host(weights) if train else None
+            gs.gs_plan_launch(plan)
+            torch.cuda.synchronize()
+            res = oracle.step(us0, es0, grads, w.rho, coeffs, c, k)
+            gi, gv = H.host(run.idx), H.host(run.vals)
+            H.compare_step(res, coeffs, [H.host(u) for u in run.us], [H.host(e) for e in run.es], gi, gv,
+                           H.host(run.est), k, H.worker_tables(run, P, r, c), H.merged_table(run, r, c))
+            if train:
+                want = w0.copy()
+                want[gi] = (w0[gi] - np.float32(lr) * gv).astype(np.float32)
+                assert np.array_equal(H.host(weights).view(np.uint32), want.view(np.uint32))
+        times = gs.gs_plan_insert_times(plan, 100)
+        assert len(times) == steps and all(t > 0 for t in times)
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()
+
+
+def test_step_plan_untimed_rejects_times(gs, H):
+    run = H.new_run(2, 4096, 3, 256, 8, 3)
+    g = [torch.zeros(4096, device="cuda") for _ in range(2)]
+    plan = gs.gs_step_plan_create(run.sketch, run.us, run.es, g, 4096, 0.9, 8, run.idx, run.vals, None, None, 0.0,
+                                  run.ws)
+    try:
+        gs.gs_plan_launch(plan)
+        with pytest.raises(gs.GsError):
+            gs.gs_plan_insert_times(plan, 4)
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()
+
+
+def test_step_plan_ring_keeps_last_launches(gs, H):
+    """More launches than the ring holds: the times of the last 1024 are returned."""
+    run = H.new_run(2, 8192, 3, 512, 16, 4)
+    g = [torch.randn(8192, device="cuda") for _ in range(2)]
+    plan = gs.gs_step_plan_create(run.sketch, run.us, run.es, g, 8192, 0.9, 16, run.idx, run.vals, None, None, 0.0,
+                                  run.ws, flags=gs.GS_PLAN_TIME_INSERT)
+    try:
+        for _ in range(1100):
+            gs.gs_plan_launch(plan)
+        times = gs.gs_plan_insert_times(plan, 2000)
+        assert len(times) == 1024 and all(t > 0 for t in times)
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()
+
+
+def test_step_host_plan(gs, H):
+    w = workloads.get_config("resnet18")
+    P, d, r, c, k, seed = 5, 300_001, 5, 4096, 300, 43
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho)
+    host = [torch.empty(d, dtype=torch.float32).pin_memory() for _ in range(P)]
+    gdev = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+    idx_h = torch.empty(k, dtype=torch.int64).pin_memory()
+    vals_h = torch.empty(k, dtype=torch.float32).pin_memory()
+    plan = gs.gs_step_host_plan_create(run.sketch, run.us, run.es, host, gdev, d, w.rho, k, idx_h, vals_h, run.ws,
+                                       flags=gs.GS_PLAN_TIME_INSERT)
+    try:
+        for t in range(3):
+            grads = workloads.make_gradients(w, t, range(P), d=d)
+            for hb, g in zip(host, grads):
+                hb.copy_(torch.from_numpy(g))
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            gs.gs_plan_launch(plan)
+            torch.cuda.current_stream().synchronize()
+            res = oracle.step(us0, es0, grads, w.rho, coeffs, c, k)
+            idx, vals = idx_h.numpy().copy(), vals_h.numpy().copy()
+            band = oracle.cell_band(res.merged_abs, coeffs, np.arange(d))
+            H.check_topk_set(idx, res.idx, res.est, band, k, d)
+            H.check_state([H.host(u) for u in run.us], [H.host(e) for e in run.es], res, idx)
+            H.check_vals(vals, idx, res.es_pre)
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()
+
+
+def test_sketched_state_plan(gs):
+    P, d, r, c, k, seed, rho, lr, rel = 4, 50_000, 5, 2048, 100, 77, 0.9, 0.05, 1e-5
+    rng = np.random.default_rng(seed)
+    co = oracle.derive_coefficients(r, seed)
+    wk = gs.gs_sketch_create(r, c, seed, P, 0)
+    U = gs.gs_sketch_create(r, c, seed, 1, 0)
+    E = gs.gs_sketch_create(r, c, seed, 1, 0)
+    gs.gs_sketch_zero(U)
+    gs.gs_sketch_zero(E)
+    gbuf = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+    ws = torch.empty(gs.gs_step_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+    idx = torch.empty(k, dtype=torch.int64, device="cuda")
+    vals = torch.empty(k, dtype=torch.float32, device="cuda")
+    weights = _dev(rng.standard_normal(d).astype(np.float32))
+    plan = gs.gs_sketched_state_plan_create(wk, U, E, gbuf, d, rho, k, idx, vals, weights, lr, ws,
+                                            flags=gs.GS_PLAN_TIME_INSERT)
+
+    def table(sk):
+        buf = np.empty(r * c, dtype=np.float32)
+        gs.gs_sketch_copy_to_host(sk, -1, buf)
+        return buf.reshape(r, c).astype(np.float64)
+
+    try:
+        AU = np.zeros((r, c))
+        AE = np.zeros((r, c))
+        for t in range(3):
+            grads = [rng.standard_normal(d).astype(np.float32) for _ in range(P)]
+            for p in range(P):
+                grads[p][rng.integers(0, d, 5)] += np.float32(25.0)
+            for b, g in zip(gbuf, grads):
+                b.copy_(torch.from_numpy(g))
+            U0, E0, w0 = table(U), table(E), weights.cpu().numpy()
+            gs.gs_plan_launch(plan)
+            torch.cuda.synchronize()
+            res = oracle.sketched_state_step(U0, E0, AU, AE, grads, rho, co, c, k, rel)
+            gi, gv = idx.cpu().numpy(), vals.cpu().numpy()
+            assert np.all(np.diff(gi) > 0) and gi.size == k
+            sym = np.setxor1d(gi, res.idx)
+            if sym.size:
+                a = np.abs(res.est)
+                kth = res.idx[np.argmin(a[res.idx])]
+                assert np.all(np.abs(a[sym] - a[kth]) <= res.band[sym] + res.band[kth])
+            assert np.all(np.abs(gv.astype(np.float64) - res.est[gi]) <= res.band[gi])
+            SD, AD = oracle.sketch_sparse(gi, gv.astype(np.float64), co, c)
+            assert np.all(np.abs(table(E) - (res.E_pre - SD)) <= rel * (res.AE_pre + AD))
+            want = w0.copy()
+            want[gi] = (w0[gi] - np.float32(lr) * gv).astype(np.float32)
+            assert np.array_equal(weights.cpu().numpy().view(np.uint32), want.view(np.uint32))
+            du = oracle.query_at(res.U_pre, co, gi)
+            _, ADu = oracle.sketch_sparse(gi, du, co, c)
+            AU, AE = res.AU_pre + ADu, res.AE_pre + AD
+        assert len(gs.gs_plan_insert_times(plan, 10)) == 3
+    finally:
+        gs.gs_plan_destroy(plan)
+        for s in (wk, U, E):
+            gs.gs_sketch_destroy(s)
