@@ -36,7 +36,7 @@ import workloads  # noqa: E402
 METRIC = "gradient coords/s through accumulate+sketch+merge+top-k at P=8; % HBM roofline"
 UNIT = "coords/s"
 K1_SOURCE = os.path.join(ROOT, "paper_2108_06004_gb300", "csrc", "k_insert.cu")
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "accumulate_insert_resnet18.md")
+PROFILE_DIR = os.path.join(ROOT, "profiles")
 CPU_SAMPLE_D = 1 << 22   # coordinates per worker in one bounded oracle step (CPU baseline)
 REF_BUDGET_S = 120.0     # oracle seconds for a whole --impl reference run
 ORACLE_S_PER_COORD = 1.7e-7  # oracle seconds per worker-coordinate (sizes the reference samples)
@@ -144,11 +144,12 @@ class ClockSampler:
 
 # ---- profile summary (ncu traffic) -------------------------------------------------------
 
-def k1_traffic_per_launch():
-    """DRAM bytes per launch of the fused accumulate+insert kernel from the committed ncu
-    summary, if that summary was taken on the current kernel source (else None)."""
+def k1_traffic_per_launch(workload: str):
+    """DRAM bytes per launch of the fused accumulate+insert kernel on this workload from the
+    committed ncu summary (profiles/accumulate_insert_<workload>.md), if there is one and it
+    was taken on the current kernel source (else None)."""
     try:
-        text = open(PROFILE_SUMMARY).read()
+        text = open(os.path.join(PROFILE_DIR, f"accumulate_insert_{workload}.md")).read()
     except OSError:
         return None
     src = hashlib.sha256(open(K1_SOURCE, "rb").read()).hexdigest()[:16]
@@ -299,7 +300,8 @@ def run_ours(args):
         else:
             gs.gs_gather_and_zero(us, es, d, idx, k, vals, stream)
 
-    for t in range(args.warmup):
+    n_warm = max(args.warmup, len(plans))  # at least W steps, and every plan launched once
+    for t in range(n_warm):
         step(t, False)
     torch.cuda.synchronize()
 
@@ -360,7 +362,7 @@ def run_ours(args):
         "row_passes": passes, "groups": groups, "algorithmic_bytes_per_worker_coord": per_wc,
         "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
         "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
-        "traffic": k1_traffic_per_launch() if variant != "sketched_state" and groups * passes == 1 else None,
+        "traffic": k1_traffic_per_launch(w.name) if variant != "sketched_state" and groups * passes == 1 else None,
         "algorithmic_bytes_per_launch": phase_bytes / (groups * passes) if passes == 1 else None,
         "algorithmic_bytes_per_phase": phase_bytes,
         "avg_launch_ms": round(sum(k1_ms) / len(k1_ms) / (groups * passes), 4),
@@ -395,7 +397,7 @@ def run_ours(args):
                 gs.gs_step_host(sk, us, es, host_pool[t % len(host_pool)], grad_dev, d, rho, k, idx_h, vals_h, ws,
                                 None, stream)
 
-        for t in range(args.warmup):
+        for t in range(max(args.warmup, len(hplans))):  # every plan once, at least W steps
             host_step(t)
         if world > 1:
             import torch.distributed as dist
@@ -436,7 +438,8 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": w.name, "variant": variant, "launch": "plan" if use_plan else "eager", "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
+        "config": {"workload": w.name, "variant": variant, "launch": "plan" if use_plan else "eager",
+                   "warmup_steps_run": n_warm, "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
                    "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
                    "l2": f"inputs larger than L2 ({P * d * 12 / 1e9:.2f} GB of g,u,e streamed per step)",
                    "d_steps_per_s": world * d * args.steps / (elapsed_ms / 1e3)},
@@ -465,6 +468,7 @@ def cpu_baseline(w, steps=1, d_s=CPU_SAMPLE_D):
     """The oracle, as it stands, on the first d_s coordinates of each worker's gradient
     (same P, r, c and rho; k scaled with d); the same unit as the metric."""
     import oracle
+    d_s = min(d_s, w.d)
     k_s = max(1, round(w.k * d_s / w.d))
     coeffs = oracle.derive_coefficients(w.r, 20210813)
     us = [np.zeros(d_s, np.float32) for _ in range(w.P)]

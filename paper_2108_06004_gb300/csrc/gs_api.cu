@@ -478,15 +478,11 @@ gs_status capture_plan(int device, int32_t flags, gs_plan** out, Body&& body) {
   const gs_status st = body(cs, marks);
   cudaGraph_t graph = nullptr;
   e = cudaStreamEndCapture(cs, &graph);
-  cudaStreamDestroy(cs);
   p->graph = graph;
-  if (st != GS_OK) {
+  if (st != GS_OK || e != cudaSuccess) {
+    cudaStreamDestroy(cs);
     plan_free(p);
-    return st;
-  }
-  if (e != cudaSuccess) {
-    plan_free(p);
-    return cuda_fail(e, "stream capture");
+    return st != GS_OK ? st : cuda_fail(e, "stream capture");
   }
   if (p->timed) {
     size_t n = 0;
@@ -507,6 +503,10 @@ gs_status capture_plan(int device, int32_t flags, gs_plan** out, Body&& body) {
     }
   }
   if (e == cudaSuccess) e = cudaGraphInstantiate(&p->exec, graph, 0);
+  // upload now, so that the first launch does not pay for it
+  if (e == cudaSuccess) e = cudaGraphUpload(p->exec, cs);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(cs);
+  cudaStreamDestroy(cs);
   if (e != cudaSuccess) {
     plan_free(p);
     return cuda_fail(e, "graph instantiation");

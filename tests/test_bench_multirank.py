@@ -53,3 +53,13 @@ def test_reference_arm_only_on_rank_zero(monkeypatch, capsys):
     args = type("A", (), {"config": "tiny-2^20", "steps": 1, "warmup": 0})()
     bench.run_reference(args)
     assert capsys.readouterr().out == ""
+
+
+def test_cpu_baseline_sample_fits_every_workload():
+    """The bounded oracle sample never asks for more coordinates than the workload has."""
+    import bench
+    import workloads
+    w = workloads.get_config("tiny-2^20")
+    cpu = bench.cpu_baseline(w, steps=1, d_s=1 << 22)
+    assert cpu["value"] > 0 and cpu["kind"] == "oracle"
+    assert f"first {w.d} coordinates" in cpu["sample"]
