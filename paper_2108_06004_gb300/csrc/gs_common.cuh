@@ -8,6 +8,8 @@
 
 #include "gs_sketch.h"
 
+#include <utility>
+
 namespace gs {
 
 constexpr uint64_t kP61 = (1ull << 61) - 1;
@@ -147,5 +149,33 @@ cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, 
                                       cudaStream_t s);
 
 inline bool is_pow2(uint32_t c) { return c && !(c & (c - 1)); }
+
+// ---- launches -----------------------------------------------------------------------
+// Every kernel of the library is launched with programmatic stream serialization (sm_90+):
+// the next kernel in the stream may be scheduled before this one has finished, and it begins
+// with grid_begin(), which waits until the grids it depends on have completed and their
+// memory is visible (griddepcontrol.wait), then lets its own successor be scheduled
+// (griddepcontrol.launch_dependents).  Launch latency and the ramp of the next grid overlap
+// the tail of the previous one; no kernel touches memory before its wait.  A kernel launched
+// after a memset, an event record or another library's kernel simply finds its wait satisfied.
+__device__ __forceinline__ void grid_begin() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 }  // namespace gs

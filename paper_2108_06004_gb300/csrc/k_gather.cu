@@ -15,6 +15,7 @@ namespace gs {
 namespace {
 
 __global__ void __launch_bounds__(kBlock) k_gather_and_zero(const __grid_constant__ GatherParams prm) {
+  grid_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < prm.k; t += stride) {
     const int64_t i = prm.idx[t];
@@ -37,6 +38,7 @@ __global__ void __launch_bounds__(kBlock) k_gather_and_zero(const __grid_constan
 __global__ void __launch_bounds__(kBlock) k_apply_update(float* __restrict__ w, int64_t d,
                                                          const int64_t* __restrict__ idx,
                                                          const float* __restrict__ vals, int64_t k, float lr) {
+  grid_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < k; t += stride) {
     const int64_t i = idx[t];
@@ -51,7 +53,7 @@ cudaError_t launch_apply_update(float* w, int64_t d, const int64_t* idx, const f
   const int64_t need = (k + kBlock - 1) / kBlock;
   const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)k_apply_update, kBlock);
   const int grid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
-  k_apply_update<<<grid, kBlock, 0, s>>>(w, d, idx, vals, k, lr);
+  launch(k_apply_update, grid, kBlock, s, w, d, idx, vals, k, lr);
   return cudaGetLastError();
 }
 
@@ -59,7 +61,7 @@ cudaError_t launch_gather_and_zero(const GatherParams& p, cudaStream_t s) {
   const int64_t need = (p.k + kBlock - 1) / kBlock;
   const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)k_gather_and_zero, kBlock);
   const int grid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
-  k_gather_and_zero<<<grid, kBlock, 0, s>>>(p);
+  launch(k_gather_and_zero, grid, kBlock, s, p);
   return cudaGetLastError();
 }
 

@@ -29,6 +29,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate(float* __restrict__ u,
                                                        float* __restrict__ e,
                                                        const float* __restrict__ g, int64_t d,
                                                        float rho, int vec) {
+  grid_begin();
   const int64_t nq = (d + 3) / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nq; q += stride) {
@@ -98,6 +99,7 @@ __device__ __forceinline__ void load_lane(const InsertParams& prm, int w, int64_
 //   POW2: c is a power of two (bucket = x & (c - 1)).
 template <int W, bool ACC, bool VEC, bool POW2>
 __global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_constant__ InsertParams prm) {
+  grid_begin();
   const int64_t d = prm.d;
   const int64_t nq = (d + 3) / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -146,6 +148,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_const
 // bound here).
 template <int W, bool ACC, bool VEC, bool POW2>
 __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_constant__ InsertParams prm) {
+  grid_begin();
   constexpr int G = W / 4;
   const int sub = threadIdx.x % G;
   const int64_t d = prm.d;
@@ -189,6 +192,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_
 // Insert one vector (prm.e[0]) into lane prm.lane of a W-wide group table.
 template <bool POW2>
 __global__ void __launch_bounds__(kBlock) k_insert_lane(const __grid_constant__ InsertParams prm, int W) {
+  grid_begin();
   const int64_t d = prm.d;
   const int64_t nq = (d + 3) / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -221,6 +225,7 @@ __global__ void __launch_bounds__(kBlock) k_insert_lane(const __grid_constant__ 
 __global__ void k_hash_eval(const __grid_constant__ HashCoeffs h, int r, uint32_t c,
                             const int64_t* __restrict__ coords, int64_t n,
                             int32_t* __restrict__ bucket_out, int8_t* __restrict__ sign_out) {
+  grid_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += stride) {
     const int64_t i = coords[t];
@@ -251,11 +256,11 @@ cudaError_t launch_ai_t(const InsertParams& p, cudaStream_t s) {
   if constexpr (W >= 4) {
     auto kern = k_accumulate_insert_coop<W, ACC, VEC, POW2>;
     const int grid = grid_for(kern, (p.d + 3) / 4 * (W / 4), kBlock);
-    kern<<<grid, kBlock, 0, s>>>(p);
+    launch(kern, grid, kBlock, s, p);
   } else {
     auto kern = k_accumulate_insert<W, ACC, VEC, POW2>;
     const int grid = grid_for(kern, (p.d + 3) / 4, kBlock);
-    kern<<<grid, kBlock, 0, s>>>(p);
+    launch(kern, grid, kBlock, s, p);
   }
   return cudaGetLastError();
 }
@@ -279,7 +284,7 @@ cudaError_t launch_accumulate(float* u, float* e, const float* g, int64_t d, flo
   const bool vec = ((reinterpret_cast<uintptr_t>(u) | reinterpret_cast<uintptr_t>(e) |
                      reinterpret_cast<uintptr_t>(g)) & 15u) == 0;
   const int grid = grid_for(k_accumulate, (d + 3) / 4, kBlock);
-  k_accumulate<<<grid, kBlock, 0, s>>>(u, e, g, d, rho, vec ? 1 : 0);
+  launch(k_accumulate, grid, kBlock, s, u, e, g, d, rho, vec ? 1 : 0);
   return cudaGetLastError();
 }
 
@@ -297,10 +302,10 @@ cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool acc, boo
 cudaError_t launch_insert_lane(const InsertParams& p, int W, cudaStream_t s) {
   if (is_pow2(p.c)) {
     const int grid = grid_for(k_insert_lane<true>, (p.d + 3) / 4, kBlock);
-    k_insert_lane<true><<<grid, kBlock, 0, s>>>(p, W);
+    launch(k_insert_lane<true>, grid, kBlock, s, p, W);
   } else {
     const int grid = grid_for(k_insert_lane<false>, (p.d + 3) / 4, kBlock);
-    k_insert_lane<false><<<grid, kBlock, 0, s>>>(p, W);
+    launch(k_insert_lane<false>, grid, kBlock, s, p, W);
   }
   return cudaGetLastError();
 }
@@ -308,7 +313,7 @@ cudaError_t launch_insert_lane(const InsertParams& p, int W, cudaStream_t s) {
 cudaError_t launch_hash_eval(const HashCoeffs& h, int r, uint32_t c, const int64_t* coords,
                              int64_t n, int32_t* bucket_out, int8_t* sign_out, cudaStream_t s) {
   const int grid = grid_for(k_hash_eval, n, kBlock);
-  k_hash_eval<<<grid, kBlock, 0, s>>>(h, r, c, coords, n, bucket_out, sign_out);
+  launch(k_hash_eval, grid, kBlock, s, h, r, c, coords, n, bucket_out, sign_out);
   return cudaGetLastError();
 }
 

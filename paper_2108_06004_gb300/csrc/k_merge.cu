@@ -43,6 +43,7 @@ __device__ __forceinline__ void load_group(const float* __restrict__ src, float*
 // registers; the rounds test a + s < P at run time.
 template <int W, int PMAX>
 __global__ void __launch_bounds__(kBlock) k_merge(const __grid_constant__ MergeParams prm) {
+  grid_begin();
   static_assert(PMAX % W == 0, "PMAX must be a multiple of W");
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int P = prm.P;
@@ -75,7 +76,7 @@ cudaError_t launch_t(const MergeParams& p, cudaStream_t s) {
   const int64_t need = (p.cells + kBlock - 1) / kBlock;
   const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)kern, kBlock);
   const int grid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
-  kern<<<grid, kBlock, 0, s>>>(p);
+  launch(kern, grid, kBlock, s, p);
   return cudaGetLastError();
 }
 

@@ -199,6 +199,7 @@ __device__ __forceinline__ void store_est(const QueryParams& prm, int64_t i0, in
 // coordinates; their hash values after the first come from the incremental form.
 template <int R>
 __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryParams prm) {
+  grid_begin();
   __shared__ uint32_t sh[kBins];
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
   __syncthreads();
@@ -244,6 +245,7 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
 
 // General path: any r <= 16 and any c (bucket by 64-bit remainder).
 __global__ void __launch_bounds__(kBlock) k_query_generic(const __grid_constant__ QueryParams prm) {
+  grid_begin();
   __shared__ uint32_t sh[kBins];
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
   __syncthreads();
@@ -308,62 +310,78 @@ __device__ __forceinline__ void load_quads(const float* __restrict__ est, int64_
 // ---- selection with candidate lists --------------------------------------------------------
 
 // One pass over est after the level-1 pick.  Keys above the level-1 bin are selected for
-// certain: their bit goes into gt_bm.  Keys inside the bin are appended to `cand` (index, key)
-// and feed the level-2 histogram; the level-2 pick follows.  A warp reserves room for all
-// candidates of its kU x 4 slots with a single atomic on the shared counter.
+// certain: their bit goes into gt_bm.  Keys inside the bin are candidates (index, key): they
+// feed the level-2 histogram and are appended to `cand`; the level-2 pick follows.  Both are
+// rare (fewer than k keys lie above the bin, and the bin is a narrow band of keys), so the
+// common path per key is a mask, a shift and a compare.  Candidates collect in a block-local
+// buffer (slots taken with a warp-aggregated shared atomic) that is copied out with one
+// global reservation per block; a block whose buffer fills up appends the rest directly
+// (warp-aggregated global atomics), which only happens for inputs with many equal keys.
 // `src` holds the keys as 32-bit words: the bits of est (kmask drops the sign) or a key array.
+constexpr int kCandBuf = 2048;
+
+__device__ __forceinline__ void cand_append(uint32_t i, uint32_t key, uint32_t* sh_n, uint2* sh_cand,
+                                            SelectState* st, uint2* __restrict__ cand) {
+  const int lane = threadIdx.x & 31;
+  uint32_t am = __activemask();
+  int leader = __ffs(am) - 1;
+  uint32_t base = 0;
+  if (lane == leader) base = atomicAdd(sh_n, (uint32_t)__popc(am));
+  base = __shfl_sync(am, base, leader);
+  const uint32_t slot = base + __popc(am & ((1u << lane) - 1u));
+  if (slot < (uint32_t)kCandBuf) {
+    sh_cand[slot] = make_uint2(i, key);
+    return;
+  }
+  am = __activemask();
+  leader = __ffs(am) - 1;
+  uint32_t gbase = 0;
+  if (lane == leader) gbase = atomicAdd(&st->ncand, (uint32_t)__popc(am));
+  gbase = __shfl_sync(am, gbase, leader);
+  cand[gbase + __popc(am & ((1u << lane) - 1u))] = make_uint2(i, key);
+}
+
 __global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ src, int64_t d, int vec, uint32_t kmask,
                                                  SelectState* st, uint32_t* hist2, uint2* __restrict__ cand,
                                                  uint32_t* gt_bm) {
+  grid_begin();
   __shared__ uint32_t sh[kBins];
+  __shared__ uint2 sh_cand[kCandBuf];
+  __shared__ uint32_t sh_n, sh_base;
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
+  if (threadIdx.x == 0) sh_n = 0;
   __syncthreads();
   const uint32_t b1 = __ldcg(&st->prefix);
   const int64_t nq = (d + 3) / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int lane = threadIdx.x & 31;
-  const uint32_t lower = (1u << lane) - 1u;
   for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += kU * stride) {
     float v[kU][4];
     int tm[kU];
     load_quads(src, d, vec, q0, stride, v, tm);
-    uint32_t keys[kU][4];
-    uint32_t slot_mask[kU][4];
-    uint32_t total = 0;
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
-      const int64_t i0 = (q0 + u * stride + lane) * 4;
+      const uint32_t i0 = (uint32_t)((q0 + u * stride + lane) * 4);
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
         const uint32_t key = __float_as_uint(v[u][t]) & kmask;
-        const bool valid = t < tm[u];
-        const uint32_t bin1 = key >> kL1Shift;
-        const int64_t i = i0 + t;
-        if (valid && bin1 > b1) atomicOr(&gt_bm[i >> 5], 1u << (i & 31));
-        keys[u][t] = key;
-        slot_mask[u][t] = __ballot_sync(kFull, valid && bin1 == b1);
-        total += __popc(slot_mask[u][t]);
-      }
-    }
-    if (total == 0) continue;  // warp-uniform
-    uint32_t base = 0;
-    if (lane == 0) base = atomicAdd(&st->ncand, total);
-    base = __shfl_sync(kFull, base, 0);
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int64_t i0 = (q0 + u * stride + lane) * 4;
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        const uint32_t m = slot_mask[u][t];
-        if (m) {
-          const bool in = (m >> lane) & 1u;
-          if (in) cand[base + __popc(m & lower)] = make_uint2((uint32_t)(i0 + t), keys[u][t]);
-          hist_add(sh, in ? ((keys[u][t] >> kL2Shift) & (kBins - 1)) : kNone);
-          base += __popc(m);
+        if (t < tm[u] && (key >> kL1Shift) >= b1) {
+          const uint32_t i = i0 + t;
+          if ((key >> kL1Shift) > b1) {
+            atomicOr(&gt_bm[i >> 5], 1u << (i & 31));
+          } else {
+            atomicAdd(&sh[(key >> kL2Shift) & (kBins - 1)], 1u);
+            cand_append(i, key, &sh_n, sh_cand, st, cand);
+          }
         }
       }
     }
   }
+  __syncthreads();
+  const uint32_t n = sh_n < (uint32_t)kCandBuf ? sh_n : (uint32_t)kCandBuf;
+  if (threadIdx.x == 0) sh_base = n ? atomicAdd(&st->ncand, n) : 0u;
+  __syncthreads();
+  for (uint32_t t = threadIdx.x; t < n; t += blockDim.x) cand[sh_base + t] = sh_cand[t];
   hist_flush(sh, hist2, kBins);
   last_block_pick(hist2, 11, st, 1, 0);
 }
@@ -371,6 +389,7 @@ __global__ void __launch_bounds__(kBlock) k_cand(const float* __restrict__ src, 
 // Level-3 histogram of the candidates that match the 22-bit prefix; the last pick gives tau.
 __global__ void __launch_bounds__(kBlock) k_cand_hist3(const uint2* __restrict__ cand, SelectState* st,
                                                        uint32_t* hist3) {
+  grid_begin();
   constexpr int kN3 = 1 << kL3Bits;
   __shared__ uint32_t sh[kN3];
   for (int b = threadIdx.x; b < kN3; b += blockDim.x) sh[b] = 0;
@@ -395,6 +414,7 @@ __global__ void __launch_bounds__(kBlock) k_cand_hist3(const uint2* __restrict__
 // Candidates above tau into gt_bm, candidates equal to tau into eq_bm.
 __global__ void __launch_bounds__(kBlock) k_cand_mark(const uint2* __restrict__ cand, const SelectState* st,
                                                       uint32_t* gt_bm, uint32_t* eq_bm) {
+  grid_begin();
   const uint32_t n = __ldcg(&st->ncand);
   const uint32_t tau = __ldcg(&st->tau);
   for (uint32_t t = blockIdx.x * blockDim.x + threadIdx.x; t < n; t += gridDim.x * blockDim.x) {
@@ -411,6 +431,7 @@ constexpr int kBmWords = kBmThreads * kBmWordsPerThread;  // 2048 words = 65536 
 __global__ void __launch_bounds__(kBmThreads) k_bm_count(const uint32_t* __restrict__ gt_bm,
                                                          const uint32_t* __restrict__ eq_bm, int64_t nbw,
                                                          uint32_t* blk_gt, uint32_t* blk_eq) {
+  grid_begin();
   const int64_t w0 = (int64_t)blockIdx.x * kBmWords + (int64_t)threadIdx.x * kBmWordsPerThread;
   uint32_t gt = 0, eq = 0;
 #pragma unroll
@@ -433,6 +454,7 @@ __global__ void __launch_bounds__(kScanThreads) k_scan(const uint32_t* __restric
                                                        const uint32_t* __restrict__ blk_eq, int64_t nblk,
                                                        const SelectState* st, uint32_t* blk_base,
                                                        uint32_t* blk_eqx) {
+  grid_begin();
   const uint32_t need_eq = __ldcg(&st->need_eq);
   uint32_t carry_gt = 0, carry_eq = 0;
   for (int64_t c0 = 0; c0 < nblk; c0 += blockDim.x) {
@@ -458,6 +480,7 @@ __global__ void __launch_bounds__(kBmThreads) k_bm_write(const uint32_t* __restr
                                                          const SelectState* st, const uint32_t* __restrict__ blk_base,
                                                          const uint32_t* __restrict__ blk_eqx,
                                                          int64_t* __restrict__ idx_out, int64_t k) {
+  grid_begin();
   const uint32_t need_eq = __ldcg(&st->need_eq);
   const uint32_t base = blk_base[blockIdx.x];
   const uint32_t eqx = blk_eqx[blockIdx.x];
@@ -505,6 +528,7 @@ __global__ void __launch_bounds__(kBmThreads) k_bm_write(const uint32_t* __restr
 __global__ void __launch_bounds__(kBlock) k_hist(const float* __restrict__ est, int64_t d, int vec,
                                                  SelectState* st, uint32_t* hist, int shift, int nbits,
                                                  int level) {
+  grid_begin();
   __shared__ uint32_t sh[kBins];
   const int nbins = 1 << nbits;
   for (int b = threadIdx.x; b < nbins; b += blockDim.x) sh[b] = 0;
@@ -567,6 +591,7 @@ template <bool VEC>
 __global__ void __launch_bounds__(kSegThreads) k_count(const float* __restrict__ est, int64_t d,
                                                        const SelectState* st, uint32_t* blk_gt,
                                                        uint32_t* blk_eq) {
+  grid_begin();
   const uint32_t tau = __ldcg(&st->tau);
   const int64_t s0 = (int64_t)blockIdx.x * kSeg;
   const int64_t s1 = s0 + kSeg < d ? s0 + kSeg : d;
@@ -597,6 +622,7 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
                                                        const SelectState* st, const uint32_t* __restrict__ blk_base,
                                                        const uint32_t* __restrict__ blk_eqx,
                                                        int64_t* __restrict__ idx_out, int64_t k) {
+  grid_begin();
   __shared__ uint32_t warp_tot[kSegWarps];
   const uint32_t tau = __ldcg(&st->tau), need_eq = __ldcg(&st->need_eq);
   const int64_t s0 = (int64_t)blockIdx.x * kSeg;
@@ -669,6 +695,7 @@ __global__ void __launch_bounds__(kSegThreads) k_write(const float* __restrict__
 
 // Sum of squares of each row of the merged table in fp64; blockIdx.y is the row.
 __global__ void __launch_bounds__(kBlock) k_row_sumsq(const float* __restrict__ T, uint32_t c, double* sumsq) {
+  grid_begin();
   __shared__ double warp_acc[kBlock / 32];
   const int j = blockIdx.y;
   const float* row = T + (size_t)j * c;
@@ -693,6 +720,7 @@ __global__ void __launch_bounds__(kBlock) k_row_sumsq(const float* __restrict__ 
 // theta = l2sq / k, the threshold of H.
 __global__ void k_heavy_theta(const double* __restrict__ sumsq, int r, int64_t k, double* theta,
                               double* l2sq_out) {
+  grid_begin();
   if (blockIdx.x != 0 || threadIdx.x != 0) return;
   double v[GS_MAX_ROWS];
   for (int j = 0; j < r; ++j) v[j] = __ldcg(&sumsq[j]);
@@ -729,6 +757,7 @@ __global__ void __launch_bounds__(kBlock) k_heavy_keys(const float* __restrict__
                                                        const double* __restrict__ theta_p, uint64_t fill_seed,
                                                        uint32_t* __restrict__ keys, uint32_t* hist1, SelectState* st,
                                                        uint32_t k) {
+  grid_begin();
   __shared__ uint32_t sh[kBins];
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
   __syncthreads();
@@ -764,7 +793,7 @@ int persistent_grid(K kernel, int64_t work_items, int block) {
 template <int R>
 cudaError_t launch_query_r(const QueryParams& p, cudaStream_t s) {
   auto kern = k_query<R>;
-  kern<<<persistent_grid(kern, (p.d + 3) / 4, kBlock), kBlock, 0, s>>>(p);
+  launch(kern, persistent_grid(kern, (p.d + 3) / 4, kBlock), kBlock, s, p);
   return cudaGetLastError();
 }
 
@@ -780,7 +809,7 @@ constexpr QueryLauncher QueryTable<Rs...>::table[sizeof...(Rs)];
 cudaError_t launch_query(const QueryParams& p, cudaStream_t s) {
   using T = QueryTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
   if (is_pow2(p.c) && p.r >= 1 && p.r <= GS_MAX_ROWS) return T::table[p.r - 1](p, s);
-  k_query_generic<<<persistent_grid(k_query_generic, p.d, kBlock), kBlock, 0, s>>>(p);
+  launch(k_query_generic, persistent_grid(k_query_generic, p.d, kBlock), kBlock, s, p);
   return cudaGetLastError();
 }
 
@@ -861,19 +890,19 @@ cudaError_t clear_selection(const Workspace& w, cudaStream_t s) {
 // Levels 2 and 3 and the ordered output, after the level-1 histogram and pick of `src` keys.
 cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint32_t kmask, int64_t d, int64_t k,
                              int64_t* idx_out, cudaStream_t s) {
-  k_cand<<<persistent_grid(k_cand, (d + 3) / 4 / kU, kBlock), kBlock, 0, s>>>(src, d, vec, kmask, w.st,
+  launch(k_cand, persistent_grid(k_cand, (d + 3) / 4 / kU, kBlock), kBlock, s, src, d, vec, kmask, w.st,
                                                                                  w.hist + kBins, w.cand, w.gt_bm);
   const int small_grid = device_info().sms;
-  k_cand_hist3<<<small_grid, kBlock, 0, s>>>(w.cand, w.st, w.hist + 2 * kBins);
-  k_cand_mark<<<small_grid, kBlock, 0, s>>>(w.cand, w.st, w.gt_bm, w.eq_bm);
+  launch(k_cand_hist3, small_grid, kBlock, s, w.cand, w.st, w.hist + 2 * kBins);
+  launch(k_cand_mark, small_grid, kBlock, s, w.cand, w.st, w.gt_bm, w.eq_bm);
   uint32_t* blk_gt = w.blk;
   uint32_t* blk_eq = blk_gt + w.nblk;
   uint32_t* blk_base = blk_eq + w.nblk;
   uint32_t* blk_eqx = blk_base + w.nblk;
   const int nb = (int)w.nblk;
-  k_bm_count<<<nb, kBmThreads, 0, s>>>(w.gt_bm, w.eq_bm, w.nbw, blk_gt, blk_eq);
-  k_scan<<<1, kScanThreads, 0, s>>>(blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx);
-  k_bm_write<<<nb, kBmThreads, 0, s>>>(w.gt_bm, w.eq_bm, w.nbw, w.st, blk_base, blk_eqx, idx_out, k);
+  launch(k_bm_count, nb, kBmThreads, s, w.gt_bm, w.eq_bm, w.nbw, blk_gt, blk_eq);
+  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx);
+  launch(k_bm_write, nb, kBmThreads, s, w.gt_bm, w.eq_bm, w.nbw, w.st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();
 }
 
@@ -914,9 +943,9 @@ cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int 
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   const int gx = (int)(((int64_t)c + kBlock - 1) / kBlock < 4 * device_info().sms ? ((int64_t)c + kBlock - 1) / kBlock
                                                                                   : 4 * device_info().sms);
-  k_row_sumsq<<<dim3(gx, r), kBlock, 0, s>>>(merged, c, sumsq);
-  k_heavy_theta<<<1, 32, 0, s>>>(sumsq, r, k, theta, l2sq_out);
-  k_heavy_keys<<<persistent_grid(k_heavy_keys, d, kBlock), kBlock, 0, s>>>(est, d, theta, fill_seed, keys, w.hist,
+  launch(k_row_sumsq, dim3(gx, r), kBlock, s, merged, c, sumsq);
+  launch(k_heavy_theta, 1, 32, s, sumsq, r, k, theta, l2sq_out);
+  launch(k_heavy_keys, persistent_grid(k_heavy_keys, d, kBlock), kBlock, s, est, d, theta, fill_seed, keys, w.hist,
                                                                            w.st, (uint32_t)k);
   return select_from_keys(w, reinterpret_cast<const float*>(keys), 1, 0xFFFFFFFFu, d, k, idx_out, s);
 }
@@ -980,14 +1009,14 @@ cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, 
   const QueryParams qp = make_query_params(merged, h, r, c, d, k, est_out, hist, st);
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   const int hgrid = persistent_grid(k_hist, (d + 3) / 4 / kU, kBlock);
-  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + kBins, kL2Shift, 11, 1);
-  k_hist<<<hgrid, kBlock, 0, s>>>(est_out, d, qp.vec, st, hist + 2 * kBins, 0, kL3Bits, 2);
+  launch(k_hist, hgrid, kBlock, s, est_out, d, qp.vec, st, hist + kBins, kL2Shift, 11, 1);
+  launch(k_hist, hgrid, kBlock, s, est_out, d, qp.vec, st, hist + 2 * kBins, 0, kL3Bits, 2);
   const int nb = (int)nseg;
-  if (qp.vec) k_count<true><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_gt, blk_eq);
-  else k_count<false><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_gt, blk_eq);
-  k_scan<<<1, kScanThreads, 0, s>>>(blk_gt, blk_eq, nseg, st, blk_base, blk_eqx);
-  if (qp.vec) k_write<true><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_base, blk_eqx, idx_out, k);
-  else k_write<false><<<nb, kSegThreads, 0, s>>>(est_out, d, st, blk_base, blk_eqx, idx_out, k);
+  if (qp.vec) launch(k_count<true>, nb, kSegThreads, s, est_out, d, st, blk_gt, blk_eq);
+  else launch(k_count<false>, nb, kSegThreads, s, est_out, d, st, blk_gt, blk_eq);
+  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, nseg, st, blk_base, blk_eqx);
+  if (qp.vec) launch(k_write<true>, nb, kSegThreads, s, est_out, d, st, blk_base, blk_eqx, idx_out, k);
+  else launch(k_write<false>, nb, kSegThreads, s, est_out, d, st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();
 }
 

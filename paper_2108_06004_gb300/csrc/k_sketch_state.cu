@@ -13,6 +13,7 @@ namespace {
 __global__ void __launch_bounds__(kBlock) k_query_at(const float* __restrict__ T, const __grid_constant__ HashCoeffs h,
                                                      int r, uint32_t c, const int64_t* __restrict__ idx, int64_t k,
                                                      float* __restrict__ out) {
+  grid_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < k; t += stride) {
     const int64_t i = idx[t];
@@ -42,6 +43,7 @@ __global__ void __launch_bounds__(kBlock) k_query_at(const float* __restrict__ T
 __global__ void __launch_bounds__(kBlock) k_add_sparse(float* __restrict__ T, const __grid_constant__ HashCoeffs h,
                                                        int r, uint32_t c, const int64_t* __restrict__ idx,
                                                        const float* __restrict__ vals, int64_t k, float scale) {
+  grid_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < k; t += stride) {
     const int64_t i = idx[t];
@@ -57,6 +59,7 @@ __global__ void __launch_bounds__(kBlock) k_add_sparse(float* __restrict__ T, co
 
 __global__ void __launch_bounds__(kBlock) k_take(const float* __restrict__ src, int64_t n, const int64_t* __restrict__ idx,
                                                  int64_t k, float* __restrict__ out) {
+  grid_begin();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < k; t += stride) {
     const int64_t i = idx[t];
@@ -75,18 +78,18 @@ int small_grid(K kernel, int64_t k) {
 
 cudaError_t launch_query_at(const float* T, const HashCoeffs& h, int r, uint32_t c, const int64_t* idx, int64_t k,
                             float* out, cudaStream_t s) {
-  k_query_at<<<small_grid(k_query_at, k), kBlock, 0, s>>>(T, h, r, c, idx, k, out);
+  launch(k_query_at, small_grid(k_query_at, k), kBlock, s, T, h, r, c, idx, k, out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_add_sparse(float* T, const HashCoeffs& h, int r, uint32_t c, const int64_t* idx, const float* vals,
                               int64_t k, float scale, cudaStream_t s) {
-  k_add_sparse<<<small_grid(k_add_sparse, k), kBlock, 0, s>>>(T, h, r, c, idx, vals, k, scale);
+  launch(k_add_sparse, small_grid(k_add_sparse, k), kBlock, s, T, h, r, c, idx, vals, k, scale);
   return cudaGetLastError();
 }
 
 cudaError_t launch_take(const float* src, int64_t n, const int64_t* idx, int64_t k, float* out, cudaStream_t s) {
-  k_take<<<small_grid(k_take, k), kBlock, 0, s>>>(src, n, idx, k, out);
+  launch(k_take, small_grid(k_take, k), kBlock, s, src, n, idx, k, out);
   return cudaGetLastError();
 }
 

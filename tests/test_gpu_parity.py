@@ -191,6 +191,27 @@ def test_query_topk(gs, H, d, r, c, k):
         run.close()
 
 
+@pytest.mark.parametrize("d,k,nonzero", [(3_000_001, 5000, False), (2_500_003, 7777, True)])
+def test_topk_large_plateau(gs, H, d, k, nonzero):
+    """Millions of equal keys: every coordinate is a selection candidate, more than any
+    block-local buffer holds.  With c = 1 and r = 1 every coordinate shares one cell, so
+    |est| is the same nonzero value everywhere; the top-k is then the k smallest indices."""
+    r, c = (1, 1) if nonzero else (5, 4096)
+    run = H.new_run(1, d, r, c, k, 3)
+    try:
+        if nonzero:
+            x = np.random.default_rng(9).standard_normal(d).astype(np.float32)
+            gs.gs_sketch_insert(run.sketch, 0, _dev(x), d)
+        gs.gs_sketch_merge_tree(run.sketch, 1)
+        ws = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        gs.gs_query_topk(run.sketch, d, k, run.idx, run.est, ws)
+        est = H.host(run.est)
+        assert np.unique(np.abs(est)).size == 1 and ((est[0] != 0) == nonzero)
+        assert np.array_equal(H.host(run.idx), np.arange(k))
+    finally:
+        run.close()
+
+
 def test_topk_all_ties_and_zeros(gs, H):
     d, r, c, k = 50_000, 5, 256, 1234
     run = H.new_run(1, d, r, c, k, 1)
