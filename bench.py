@@ -369,10 +369,13 @@ def run_ours(args):
         "avg_phase_ms": round(sum(k1_ms) / len(k1_ms), 4),
         "timed_phases": len(k1_ms),
         "timing": "event-record nodes inside the step's CUDA graph" if use_plan else "CUDA events around the call",
-        "co_bound": {"kind": "l2_reductions, one 32-byte request per cell update (W=8)",
+        "co_bound": {"kind": "SM->L2 payload: cell reductions (4*r B per worker-coordinate) + u, e stores "
+                             "(8 B per worker-coordinate; none for the sketched state)",
                      "cell_updates_per_phase": cells,
                      "achieved_G_cells_per_s": round(cells / phase_s / 1e9, 1),
-                     "probe_peak_G_cells_per_s": 134.5},
+                     "probe_peak_G_cells_per_s": 134.5,
+                     "sm_to_l2_payload_GBps": round(P * d * (4 * r + (0 if variant == "sketched_state" else 8))
+                                                    / phase_s / 1e9, 1)},
         "step_share": round(sum(k1_ms) / elapsed_ms, 3),
     }
 
