@@ -362,6 +362,7 @@ def run_ours(args):
         "row_passes": passes, "groups": groups, "algorithmic_bytes_per_worker_coord": per_wc,
         "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
         "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
+        "frac_of_nominal_8000_GBps": round(k1_gbs / 8000.0, 4),
         "traffic": k1_traffic_per_launch(w.name) if variant != "sketched_state" and groups * passes == 1 else None,
         "algorithmic_bytes_per_launch": phase_bytes / (groups * passes) if passes == 1 else None,
         "algorithmic_bytes_per_phase": phase_bytes,

@@ -193,3 +193,32 @@ def test_sketched_state_plan(gs):
         gs.gs_plan_destroy(plan)
         for s in (wk, U, E):
             gs.gs_sketch_destroy(s)
+
+
+def test_step_plan_resnet18_full_size(gs, H):
+    """The launch configuration bench.py times: the ResNet-18-sized workload (d = 11,173,962,
+    P = 8, r = 5, c = 2^17, k = 11,200) stepped through a plan, two steps, every output
+    compared with the oracle."""
+    w = workloads.get_config("resnet18")
+    P, d, r, c, k, seed = w.P, w.d, w.r, w.c, w.k, 20210813
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho)
+    gbuf = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+    plan = gs.gs_step_plan_create(run.sketch, run.us, run.es, gbuf, d, w.rho, k, run.idx, run.vals, run.est,
+                                  flags=gs.GS_PLAN_TIME_INSERT, workspace=run.ws)
+    try:
+        for t in range(2):
+            grads = workloads.make_gradients(w, t, range(P))
+            for b, g in zip(gbuf, grads):
+                b.copy_(torch.from_numpy(g))
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            gs.gs_plan_launch(plan)
+            torch.cuda.synchronize()
+            res = oracle.step(us0, es0, grads, w.rho, coeffs, c, k)
+            H.compare_step(res, coeffs, [H.host(u) for u in run.us], [H.host(e) for e in run.es], H.host(run.idx),
+                           H.host(run.vals), H.host(run.est), k, H.worker_tables(run, P, r, c),
+                           H.merged_table(run, r, c))
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()
