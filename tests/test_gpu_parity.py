@@ -159,6 +159,49 @@ def test_accumulate_insert_merge(gs, H, P, W, d, r, c, passes):
         run.close()
 
 
+def test_accumulate_insert_unaligned(gs, H):
+    """Vectors that start 4 bytes past a 16-byte boundary take the scalar load path of the
+    fused kernel; the state stays bit-exact and the tables agree with the oracle."""
+    P, d, r, c, seed = 5, 100_003, 5, 4096, 77
+    rng = np.random.default_rng(seed)
+    coeffs = oracle.derive_coefficients(r, seed)
+    sk = gs.gs_sketch_create(r, c, seed, P, 0)
+    try:
+        bufs = [[torch.zeros(d + 4, dtype=torch.float32, device="cuda") for _ in range(3)] for _ in range(P)]
+        views = [[b[1:d + 1] for b in trio] for trio in bufs]
+        host = []
+        for p in range(P):
+            u, e, g = [(rng.standard_normal(d) * 1e-2).astype(np.float32) for _ in range(3)]
+            for v, x in zip(views[p], (u, e, g)):
+                v.copy_(torch.from_numpy(x))
+            host.append((u, e, g))
+        gs.gs_sketch_zero(sk)
+        gs.gs_accumulate_insert(sk, 0, [v[0] for v in views], [v[1] for v in views], [v[2] for v in views], d, 0.9)
+        gs.gs_sketch_merge_tree(sk, P)
+        torch.cuda.synchronize()
+        Ts, As = [], []
+        for p in range(P):
+            u1, e1 = oracle.accumulate(*host[p], 0.9)
+            assert np.array_equal(views[p][0].cpu().numpy().view(np.uint32), u1.view(np.uint32))
+            assert np.array_equal(views[p][1].cpu().numpy().view(np.uint32), e1.view(np.uint32))
+            T, A = oracle.sketch(e1, coeffs, c)
+            buf = np.empty(r * c, dtype=np.float32)
+            gs.gs_sketch_copy_to_host(sk, p, buf)
+            H.check_cells(buf.reshape(r, c), T, A, f"worker {p}")
+            Ts.append(T)
+            As.append(A)
+        buf = np.empty(r * c, dtype=np.float32)
+        gs.gs_sketch_copy_to_host(sk, -1, buf)
+        H.check_cells(buf.reshape(r, c), oracle.merge_tree(Ts), oracle.merge_tree(As), "merged")
+        # the guard words around each view are untouched
+        for trio in bufs:
+            for b in trio[:2]:
+                edge = b.cpu().numpy()
+                assert edge[0] == 0 and np.all(edge[d + 1:] == 0)
+    finally:
+        gs.gs_sketch_destroy(sk)
+
+
 # ---- steps 4-5 ---------------------------------------------------------------------------
 
 @pytest.mark.parametrize("d,r,c,k", [(1, 5, 64, 1), (10, 3, 1, 4), (1000, 1, 1, 1000), (100_003, 5, 4096, 1),
@@ -226,7 +269,8 @@ def test_topk_all_ties_and_zeros(gs, H):
 
 # ---- step 6 ------------------------------------------------------------------------------
 
-@pytest.mark.parametrize("P,d,k", [(1, 10, 10), (4, 1_000_003, 1000), (64, 20_000, 777)])
+@pytest.mark.parametrize("P,d,k", [(1, 10, 10), (2, 1001, 57), (3, 5003, 100), (4, 1_000_003, 1000),
+                                   (9, 20_001, 333), (17, 10_007, 99), (33, 12_345, 500), (64, 20_000, 777)])
 def test_gather_and_zero(gs, P, d, k):
     rng = np.random.default_rng(P)
     us = [(rng.standard_normal(d)).astype(np.float32) for _ in range(P)]
@@ -291,7 +335,8 @@ def test_steps_tiny_config(gs, H):
     _run_steps(gs, H, w, w.d, w.steps)
 
 
-@pytest.mark.parametrize("P,r,c,k,W", [(5, 4, 1000, 777, 0), (6, 3, 4099, 50, 2), (3, 5, 1 << 12, 1, 1)])
+@pytest.mark.parametrize("P,r,c,k,W", [(5, 4, 1000, 777, 0), (6, 3, 4099, 50, 2), (3, 5, 1 << 12, 1, 1),
+                                       (9, 5, 2048, 100, 0)])
 def test_steps_ragged(gs, H, P, r, c, k, W):
     w = workloads.get_config("resnet18")
     _run_steps(gs, H, w, 100_003, 2, c=c, k=k, r=r, P=P, group_width=W)
