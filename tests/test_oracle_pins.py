@@ -15,8 +15,6 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle import countsketch as cs
-from oracle import gssgd
 
 P61 = (1 << 61) - 1
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
