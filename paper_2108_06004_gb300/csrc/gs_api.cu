@@ -68,25 +68,29 @@ void derive_coefficients(int r, uint64_t seed, gs::HashCoeffs& h) {
   }
 }
 
-// The slice of a group table that one insert pass updates is kept within this many bytes, so
-// that the table stays resident in the 126 MB L2 while g, u and e stream past it.
-constexpr size_t kL2BudgetBytes = size_t(64) << 20;
+// L2 budgets (GB300: 126 MB of L2 in two halves).  A group's table row must fit kRowBudget,
+// else the group is narrowed; one insert pass updates at most kPassBudget of table, so that
+// the slice stays resident in L2 while g, u and e stream past it.  Measured on the VGG-16 and
+// BERT-large workloads: a 64 MB slice per pass is slower than a 32 MB one (L2 contention),
+// and 96 MB thrashes; 8-wide groups with one 64 MB row per pass beat 4-wide groups.
+constexpr size_t kRowBudget = size_t(64) << 20;
+constexpr size_t kPassBudget = size_t(48) << 20;
 
 // Widest group (up to 16, not wider than the worker count rounded up to a power of two) whose
-// single table row fits the budget.  16-wide groups are used only when the whole group table
-// fits in one pass: their 64-byte cells halve the reduction requests, but a 16-wide table
+// single table row fits the row budget.  16-wide groups are used only when the whole group
+// table fits one pass: their 64-byte cells halve the reduction requests, but a 16-wide table
 // that needs row passes re-reads e more often than two 8-wide groups do (measured slower).
 int choose_group_width(int r, int c, int workers) {
   int W = 1;
   while (W < workers && W < gs::kMaxGroup) W *= 2;
-  if (W == 16 && (size_t)r * (size_t)c * 16 * sizeof(float) > kL2BudgetBytes) W = 8;
-  while (W > 1 && (size_t)c * (size_t)W * sizeof(float) > kL2BudgetBytes) W /= 2;
+  if (W == 16 && (size_t)r * (size_t)c * 16 * sizeof(float) > kPassBudget) W = 8;
+  while (W > 1 && (size_t)c * (size_t)W * sizeof(float) > kRowBudget) W /= 2;
   return W;
 }
 
 int choose_rows_per_pass(int r, int c, int W) {
   const size_t row_bytes = (size_t)c * (size_t)W * sizeof(float);
-  size_t n = kL2BudgetBytes / row_bytes;
+  size_t n = kPassBudget / row_bytes;
   if (n < 1) n = 1;
   if (n > (size_t)r) n = (size_t)r;
   return (int)n;

@@ -112,9 +112,10 @@ def test_single_vector_insert(gs, H, W, worker, P):
 @pytest.mark.parametrize("P,W,d,r,c,passes", [(1, 1, 70_001, 3, 1 << 10, 1), (3, 4, 123_457, 5, 1000, 1),
                                               (5, 8, 200_003, 4, 1 << 13, 1), (8, 2, 65_536, 5, 1 << 12, 1),
                                               (8, 8, 400_000, 7, 1 << 14, 1), (16, 8, 50_001, 5, 777, 1),
-                                              (8, 0, 200_003, 3, 1 << 21, 3), (6, 0, 150_001, 5, 1 << 20, 3),
-                                              (4, 0, 100_001, 7, 1 << 21, 4), (16, 16, 90_001, 5, 1 << 12, 1),
-                                              (13, 0, 80_003, 3, 1 << 20, 2), (16, 0, 70_001, 5, 1 << 16, 1), (20, 16, 60_001, 4, 3001, 1)])
+                                              (8, 0, 200_003, 3, 1 << 21, 3), (6, 0, 150_001, 5, 1 << 20, 5),
+                                              (4, 0, 100_001, 7, 1 << 21, 7), (16, 16, 90_001, 5, 1 << 12, 1),
+                                              (13, 0, 80_003, 3, 1 << 20, 3), (16, 0, 70_001, 5, 1 << 16, 1), (20, 16, 60_001, 4, 3001, 1),
+                                              (8, 0, 90_001, 7, 1 << 19, 3)])
 def test_accumulate_insert_merge(gs, H, P, W, d, r, c, passes):
     seed = P * 1000 + W
     rng = np.random.default_rng(seed)
