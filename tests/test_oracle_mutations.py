@@ -74,6 +74,101 @@ def test_pin_catches_mutation(monkeypatch, name, bad, pin, kw):
         pin(**kw)
 
 
+# ---- the later oracle functions (weight update, HEAVYMIX, sketched state) -----------------
+
+_REAL = {n: getattr(gssgd, n) for n in ("apply_update", "gather_and_zero", "heavymix_select",
+                                         "sketched_state_step", "merge_schedule")}
+_REAL["derive_coefficients"] = cs.derive_coefficients
+_REAL["splitmix64_at"] = cs.splitmix64_at
+
+
+def _apply_update_fused(w, idx, vals, lr):
+    out = np.array(w, dtype=np.float32, copy=True)
+    idx = np.asarray(idx)
+    v = np.asarray(vals, dtype=np.float64)
+    out[idx] = (out[idx].astype(np.float64) - np.float64(np.float32(lr)) * v).astype(np.float32)  # one rounding
+    return out
+
+
+def _apply_update_ascent(w, idx, vals, lr):
+    return _REAL["apply_update"](w, idx, -np.asarray(vals, dtype=np.float32), lr)
+
+
+def _gather_keeps_momentum(us, es, idx):
+    vals, _, es2 = _REAL["gather_and_zero"](us, es, idx)
+    return vals, [np.array(u, copy=True) for u in us], es2
+
+
+def _gather_sums_momentum(us, es, idx):
+    _, us2, es2 = _REAL["gather_and_zero"](us, es, idx)
+    return np.sum([u[np.asarray(idx)].astype(np.float64) for u in us], axis=0), us2, es2
+
+
+def _merge_schedule_first_idles(P):
+    rounds, step = [], 1
+    while step < P:
+        parts = list(range(0, P, step))
+        if len(parts) % 2:
+            parts = parts[1:]          # the smallest id sits the round out
+        rounds.append([(parts[m], parts[m + 1]) for m in range(0, len(parts) - 1, 2)])
+        step *= 2
+    return rounds
+
+
+def _heavymix_threshold_on_abs(est, l2sq, k, fill_seed):
+    # |est| >= l2sq / k in place of est^2 >= l2sq / k
+    return _REAL["heavymix_select"](est, k * (l2sq / k) ** 2, k, fill_seed)
+
+
+def _splitmix64_at_off_by_one(seed, idx):
+    return _REAL["splitmix64_at"](seed, np.asarray(idx, dtype=np.uint64) + np.uint64(1))
+
+
+def _coefficients_draw_order(r, seed):
+    a, b, a2, b2 = _REAL["derive_coefficients"](r, seed)
+    return a, a2, b, b2                # draws taken as a, a', b, b'
+
+
+def _sketched_state_keeps_momentum(U, E, AU, AE, gs, rho, coeffs, c, k, rel=1e-5):
+    res = _REAL["sketched_state_step"](U, E, AU, AE, gs, rho, coeffs, c, k, rel)
+    res.U = res.U_pre                  # the extracted mass not removed from U
+    return res
+
+
+def _sketched_state_error_from_s(U, E, AU, AE, gs, rho, coeffs, c, k, rel=1e-5):
+    res = _REAL["sketched_state_step"](U, E, AU, AE, gs, rho, coeffs, c, k, rel)
+    res.E = res.E - res.U_pre + res.S  # E <- E + S in place of E + U
+    return res
+
+
+LATER = [
+    ("apply_update", _apply_update_fused, pins.test_apply_update_equals_numpy_fp32, {}),
+    ("apply_update", _apply_update_ascent, pins.test_apply_update_closed_form, {}),
+    ("gather_and_zero", _gather_keeps_momentum, pins.test_gather_and_zero_conservation, {}),
+    ("gather_and_zero", _gather_sums_momentum, pins.test_gather_and_zero_conservation, {}),
+    ("merge_schedule", _merge_schedule_first_idles, pins.test_merge_schedule_structure, {}),
+    ("heavymix_select", _heavymix_threshold_on_abs, pins.test_heavymix_select_brute_force_threshold_on_the_square,
+     {}),
+    ("splitmix64_at", _splitmix64_at_off_by_one, pins.test_splitmix64_counter_form_matches_stream, {}),
+    ("derive_coefficients", _coefficients_draw_order, pins.test_coefficients_ranges_and_order, {}),
+    ("sketched_state_step", _sketched_state_keeps_momentum,
+     pins.test_sketched_state_removal_and_momentum_closed_form, {}),
+    ("sketched_state_step", _sketched_state_error_from_s,
+     pins.test_sketched_state_removal_and_momentum_closed_form, {}),
+]
+
+
+@pytest.mark.parametrize("name,bad,pin,kw", LATER, ids=[m[1].__name__ for m in LATER])
+def test_pin_catches_mutation_in_later_functions(monkeypatch, name, bad, pin, kw):
+    # patched where the pins call it and where other oracle functions call it
+    monkeypatch.setattr(oracle, name, bad)
+    for mod in (gssgd, cs):
+        if hasattr(mod, name):
+            monkeypatch.setattr(mod, name, bad)
+    with pytest.raises(AssertionError):
+        pin(**kw)
+
+
 def test_pin_catches_wrong_modulus(monkeypatch):
     monkeypatch.setattr(cs, "_affine_mod_p", _affine_mod_2_61)
     with pytest.raises(AssertionError):

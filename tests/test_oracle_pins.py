@@ -40,7 +40,11 @@ def test_coefficients_ranges_and_order():
     gen = oracle.splitmix64(7)
     draws = [next(gen) for _ in range(8)]
     a, b, a2, b2 = oracle.derive_coefficients(2, 7)
-    assert a[1] == 1 + draws[4] % (P61 - 1) and b2[0] == draws[3] % P61
+    for j in range(2):
+        assert a[j] == 1 + draws[4 * j] % (P61 - 1)
+        assert b[j] == draws[4 * j + 1] % P61
+        assert a2[j] == 1 + draws[4 * j + 2] % (P61 - 1)
+        assert b2[j] == draws[4 * j + 3] % P61
     assert oracle.derive_coefficients(3, 5) != oracle.derive_coefficients(3, 6)
 
 
@@ -428,6 +432,24 @@ def test_heavymix_random_fill_brute_force():
     xi = {i: int(oracle.splitmix64_at(seed, [i])[0]) >> 33 for i in range(d)}
     nh = sorted((i for i in range(d) if i not in set(h)), key=lambda i: (xi[i], i))
     assert sorted(h + nh[: k - len(h)]) == idx.tolist()
+
+
+def test_heavymix_select_brute_force_threshold_on_the_square():
+    """H = {i : est_i^2 >= l2sq / k}, written out per coordinate, with estimates on both
+    sides of sqrt(l2sq / k) and of l2sq / k itself (where a threshold on |est| would differ),
+    and the fill by (xi_i, i) over the rest."""
+    est = np.array([3.0, -2.0, 1.9, 2.5, -0.7, 0.1, 4.5, -3.9, 0.05, 1.0, -2.1, 0.3])
+    d = est.size
+    for k, l2sq, seed in [(3, 12.0, 0), (4, 16.0, 9), (5, 20.0, 77), (2, 8.0, 2**64 - 5), (6, 3.0, 1)]:
+        thr = l2sq / k
+        h = [i for i in range(d) if est[i] * est[i] >= thr]
+        if len(h) >= k:
+            want = sorted(sorted(h, key=lambda i: (-abs(est[i]), i))[:k])
+        else:
+            xi = {i: int(oracle.splitmix64_at(seed, [i])[0]) >> 33 for i in range(d)}
+            rest = sorted((i for i in range(d) if i not in h), key=lambda i: (xi[i], i))
+            want = sorted(h + rest[: k - len(h)])
+        assert oracle.heavymix_select(est, l2sq, k, seed).tolist() == want
 
 
 def test_heavymix_fill_is_uniform():
