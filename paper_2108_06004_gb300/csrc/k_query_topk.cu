@@ -11,7 +11,12 @@
 // smallest index.  Output indices are ascending.
 //
 // With a caller workspace (gs_query_topk):
-//   k_query       est_i for every i (fp32) + level-1 histogram + pick
+//   k_query       est_i for every i (fp32) + level-1 histogram + pick; when the estimate stays
+//                 in the workspace, a coordinate whose first r/2 + 1 rows all lie below the
+//                 prune key (from the sketch's previous query) skips its other rows and stores
+//                 -0.0 (see below)
+//   k_repair      runs only if the level-1 pick fell below the prune key: recomputes every
+//                 -0.0 estimate in full, rebuilds the level-1 histogram and picks again
 //   k_cand        one pass over est: keys above the picked level-1 bin are selected for
 //                 certain and set their bit in a d-bit bitmap; keys inside the bin become
 //                 candidates (index, key) and feed the level-2 histogram + pick
@@ -46,6 +51,8 @@ struct SelectState {
   uint32_t found;    // bit l set when level l found its bin
   uint32_t ncand;    // candidates appended by k_cand
   uint32_t done[3];  // CTAs finished per level (for the last-CTA pick)
+  uint32_t prune_key;  // the key below which k_query skipped rows (0: none)
+  uint32_t done_r;     // CTAs finished in k_repair
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -143,11 +150,12 @@ __device__ void pick_bins(const uint32_t* hist, int nbits, SelectState* st, int 
 
 // Called by every CTA after its histogram atomics: the last CTA to arrive does the pick.
 __device__ __forceinline__ void last_block_pick(const uint32_t* hist, int nbits, SelectState* st, int level,
-                                                uint32_t k_init) {
+                                                uint32_t k_init, uint32_t* counter = nullptr) {
   __shared__ uint32_t am_last;
   __threadfence();
   __syncthreads();
-  if (threadIdx.x == 0) am_last = (atomicAdd(&st->done[level], 1u) == gridDim.x - 1) ? 1u : 0u;
+  if (threadIdx.x == 0)
+    am_last = (atomicAdd(counter ? counter : &st->done[level], 1u) == gridDim.x - 1) ? 1u : 0u;
   __syncthreads();
   if (am_last) {
     __threadfence();
@@ -181,8 +189,28 @@ struct QueryParams {
   uint32_t c, cmask;
   int32_t vec;        // est 16-byte aligned
   int32_t hist_on;    // build the level-1 histogram of |est| keys and pick
+  int32_t prune;      // skip rows below the prune key (estimate internal to the workspace)
+  uint32_t* qstate;   // the sketch's record of its last query: d (two words), k, tau key
   HashCoeffs h;
 };
+
+// Row pruning.  The median of r values lies between the least and the largest of any
+// r/2 + 1 of them (for even r both middle values do, and so does their fp32 mean).  So a
+// coordinate whose first r/2 + 1 signed cells all have |v| < t has |est| < t and cannot be
+// among the top k when t is at most the k-th largest |est|.  The prune key is 0.9 times the
+// k-th largest key of the sketch's previous query with the same d and k, rounded down to a
+// level-1 bin edge: whether it was safe is then exactly whether the level-1 pick lands in
+// that bin or above, which k_repair checks.
+constexpr uint32_t kPrunedBits = 0x80000000u;  // -0.0f: the stored estimate of a pruned coordinate
+
+__device__ __forceinline__ uint32_t prune_key_of(const QueryParams& prm) {
+  if (!prm.prune) return 0u;
+  const uint32_t dl = __ldcg(&prm.qstate[0]), dh = __ldcg(&prm.qstate[1]);
+  const uint32_t kk = __ldcg(&prm.qstate[2]), tk = __ldcg(&prm.qstate[3]);
+  if (dl != (uint32_t)prm.d || dh != (uint32_t)((uint64_t)prm.d >> 32) || kk != prm.k) return 0u;
+  if (tk == 0u || tk >= 0x7F800000u) return 0u;
+  return key_of(0.9f * __uint_as_float(tk)) & ~((1u << kL1Shift) - 1u);
+}
 
 __device__ __forceinline__ void store_est(const QueryParams& prm, int64_t i0, int tmax,
                                           const float (&m)[4]) {
@@ -206,6 +234,9 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
   const int64_t d = prm.d, nq = (d + 3) / 4;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int lane = threadIdx.x & 31;
+  const uint32_t pk = prune_key_of(prm);
+  if (prm.prune && blockIdx.x == 0 && threadIdx.x == 0) prm.st->prune_key = pk;
+  constexpr int kF = R / 2 + 1;  // rows that bound the median
   for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += stride) {
     const int64_t q = q0 + lane;
     const int64_t i0 = q * 4;
@@ -214,7 +245,7 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
     if (tmax > 0) {
       float v[4][R];
 #pragma unroll
-      for (int j = 0; j < R; ++j) {
+      for (int j = 0; j < kF; ++j) {
         uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
         uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
         const float* row = prm.T + (size_t)j * prm.c;
@@ -228,8 +259,31 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
           }
         }
       }
+      bool need[4];
 #pragma unroll
-      for (int t = 0; t < 4; ++t) m[t] = median_of<R>(v[t]);
+      for (int t = 0; t < 4; ++t) {
+        bool below = pk != 0u;
+#pragma unroll
+        for (int j = 0; j < kF; ++j) below = below && key_of(v[t][j]) < pk;
+        need[t] = !below;
+      }
+#pragma unroll
+      for (int j = kF; j < R; ++j) {
+        uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+        uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
+        const float* row = prm.T + (size_t)j * prm.c;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          v[t][j] = 0.f;
+          if (t < tmax) {
+            if (need[t]) v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
+            x = step61(x, prm.h.a[j]);
+            y = step61(y, prm.h.a2[j]);
+          }
+        }
+      }
+#pragma unroll
+      for (int t = 0; t < 4; ++t) m[t] = need[t] ? median_of<R>(v[t]) : __uint_as_float(kPrunedBits);
       store_est(prm, i0, tmax, m);
     }
     if (prm.hist_on) {
@@ -241,6 +295,46 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
     hist_flush(sh, prm.hist, kBins);
     last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
   }
+}
+
+// Runs after k_query.  If the level-1 pick landed in the prune key's bin or above, the k-th
+// largest |est| is at least the prune key and pruning changed nothing the selection sees: the
+// kernel returns at once.  Otherwise every stored -0.0 (each pruned coordinate, and any
+// genuine -0.0, which recomputes to itself) gets its full median, the level-1 histogram is
+// rebuilt from all estimates into hist_r, and the level-1 pick is made again.
+template <int R>
+__global__ void __launch_bounds__(kBlock) k_repair(const __grid_constant__ QueryParams prm, uint32_t* hist_r) {
+  grid_begin();
+  const uint32_t pk = __ldcg(&prm.st->prune_key);
+  if (pk == 0u || __ldcg(&prm.st->prefix) >= (pk >> kL1Shift)) return;  // uniform over the grid
+  __shared__ uint32_t sh[kBins];
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
+  __syncthreads();
+  const int64_t d = prm.d;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int lane = threadIdx.x & 31;
+  for (int64_t base = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); base < d; base += stride) {
+    const int64_t i = base + lane;
+    uint32_t bin = kNone;
+    if (i < d) {
+      float e = prm.est[i];
+      if (__float_as_uint(e) == kPrunedBits) {
+        float v[R];
+#pragma unroll
+        for (int j = 0; j < R; ++j) {
+          const uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i);
+          const uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i);
+          v[j] = apply_sign(__ldg(prm.T + (size_t)j * prm.c + ((uint32_t)x & prm.cmask)), signbit_of(y));
+        }
+        e = median_of<R>(v);
+        prm.est[i] = e;
+      }
+      bin = key_of(e) >> kL1Shift;
+    }
+    hist_add(sh, bin);
+  }
+  hist_flush(sh, hist_r, kBins);
+  last_block_pick(hist_r, 11, prm.st, 0, prm.k, &prm.st->done_r);
 }
 
 // General path: any r <= 16 and any c (bucket by 64-bit remainder).
@@ -453,9 +547,16 @@ __global__ void __launch_bounds__(kBmThreads) k_bm_count(const uint32_t* __restr
 __global__ void __launch_bounds__(kScanThreads) k_scan(const uint32_t* __restrict__ blk_gt,
                                                        const uint32_t* __restrict__ blk_eq, int64_t nblk,
                                                        const SelectState* st, uint32_t* blk_base,
-                                                       uint32_t* blk_eqx) {
+                                                       uint32_t* blk_eqx, uint32_t* qstate, int64_t d,
+                                                       uint32_t k) {
   grid_begin();
   const uint32_t need_eq = __ldcg(&st->need_eq);
+  if (qstate && threadIdx.x == 0) {  // the sketch's record of this query, for the next one's prune key
+    qstate[0] = (uint32_t)d;
+    qstate[1] = (uint32_t)((uint64_t)d >> 32);
+    qstate[2] = k;
+    qstate[3] = __ldcg(&st->tau);
+  }
   uint32_t carry_gt = 0, carry_eq = 0;
   for (int64_t c0 = 0; c0 < nblk; c0 += blockDim.x) {
     const int64_t b = c0 + threadIdx.x;
@@ -806,6 +907,26 @@ struct QueryTable {
 template <int... Rs>
 constexpr QueryLauncher QueryTable<Rs...>::table[sizeof...(Rs)];
 
+template <int R>
+cudaError_t launch_repair_r(const QueryParams& p, uint32_t* hist_r, cudaStream_t s) {
+  auto kern = k_repair<R>;
+  // one CTA per SM: the kernel almost always returns at once, and a repair is rare
+  launch(kern, device_info().sms, kBlock, s, p, hist_r);
+  return cudaGetLastError();
+}
+
+typedef cudaError_t (*RepairLauncher)(const QueryParams&, uint32_t*, cudaStream_t);
+
+template <int... Rs>
+struct RepairTable {
+  static constexpr RepairLauncher table[sizeof...(Rs)] = {&launch_repair_r<Rs>...};
+};
+template <int... Rs>
+constexpr RepairLauncher RepairTable<Rs...>::table[sizeof...(Rs)];
+
+// Pruning applies on the fast path (c a power of two) with at least three rows.
+bool can_prune(int r, uint32_t c) { return is_pow2(c) && r >= 3 && r <= GS_MAX_ROWS; }
+
 cudaError_t launch_query(const QueryParams& p, cudaStream_t s) {
   using T = QueryTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
   if (is_pow2(p.c) && p.r >= 1 && p.r <= GS_MAX_ROWS) return T::table[p.r - 1](p, s);
@@ -827,6 +948,8 @@ QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, u
   qp.cmask = c - 1;
   qp.vec = (reinterpret_cast<uintptr_t>(est) & 15u) == 0 ? 1 : 0;
   qp.hist_on = 1;
+  qp.prune = 0;
+  qp.qstate = nullptr;
   qp.h = h;
   return qp;
 }
@@ -834,7 +957,7 @@ QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, u
 // Layout of the caller's workspace for the candidate pipeline.
 struct Workspace {
   float* est;         // d
-  uint32_t* hist;     // 3 * kBins
+  uint32_t* hist;     // 4 * kBins: levels 1-3, and level 1 again for k_repair
   SelectState* st;
   uint2* cand;        // d (index, key) pairs: room for every coordinate
   uint32_t* gt_bm;    // nbw words
@@ -851,7 +974,7 @@ Workspace carve(void* base, int64_t d) {
   w.est = reinterpret_cast<float*>(p);
   p += align256((size_t)d * sizeof(float));
   w.hist = reinterpret_cast<uint32_t*>(p);
-  p += align256(3 * kBins * sizeof(uint32_t));
+  p += align256(4 * kBins * sizeof(uint32_t));
   w.st = reinterpret_cast<SelectState*>(p);
   p += align256(sizeof(SelectState));
   w.cand = reinterpret_cast<uint2*>(p);
@@ -870,7 +993,7 @@ size_t query_topk_workspace_bytes(int64_t d, int64_t k) {
   (void)k;
   const int64_t nbw = (d + 31) / 32;
   const int64_t nblk = (nbw + kBmWords - 1) / kBmWords;
-  return align256((size_t)d * sizeof(float)) + align256(3 * kBins * sizeof(uint32_t)) +
+  return align256((size_t)d * sizeof(float)) + align256(4 * kBins * sizeof(uint32_t)) +
          align256(sizeof(SelectState)) + align256((size_t)d * sizeof(uint2)) +
          2 * align256((size_t)nbw * sizeof(uint32_t)) + align256((size_t)nblk * 4 * sizeof(uint32_t));
 }
@@ -879,7 +1002,7 @@ namespace {
 
 // Histograms, state and both bitmaps back to zero.
 cudaError_t clear_selection(const Workspace& w, cudaStream_t s) {
-  cudaError_t err = cudaMemsetAsync(w.hist, 0, 3 * kBins * sizeof(uint32_t), s);
+  cudaError_t err = cudaMemsetAsync(w.hist, 0, 4 * kBins * sizeof(uint32_t), s);
   if (err == cudaSuccess) err = cudaMemsetAsync(w.st, 0, sizeof(SelectState), s);
   // the two bitmaps are adjacent: clear both at once
   if (err == cudaSuccess)
@@ -889,7 +1012,7 @@ cudaError_t clear_selection(const Workspace& w, cudaStream_t s) {
 
 // Levels 2 and 3 and the ordered output, after the level-1 histogram and pick of `src` keys.
 cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint32_t kmask, int64_t d, int64_t k,
-                             int64_t* idx_out, cudaStream_t s) {
+                             int64_t* idx_out, cudaStream_t s, uint32_t* qstate = nullptr) {
   launch(k_cand, persistent_grid(k_cand, (d + 3) / 4 / kU, kBlock), kBlock, s, src, d, vec, kmask, w.st,
                                                                                  w.hist + kBins, w.cand, w.gt_bm);
   const int small_grid = device_info().sms;
@@ -901,7 +1024,7 @@ cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint
   uint32_t* blk_eqx = blk_base + w.nblk;
   const int nb = (int)w.nblk;
   launch(k_bm_count, nb, kBmThreads, s, w.gt_bm, w.eq_bm, w.nbw, blk_gt, blk_eq);
-  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx);
+  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx, qstate, d, (uint32_t)k);
   launch(k_bm_write, nb, kBmThreads, s, w.gt_bm, w.eq_bm, w.nbw, w.st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();
 }
@@ -910,15 +1033,22 @@ cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint
 
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, cudaStream_t s) {
+                              void* workspace, cudaStream_t s, uint32_t* qstate) {
   Workspace w = carve(workspace, d);
   float* est = est_out ? est_out : w.est;
   cudaError_t err = clear_selection(w, s);
   if (err != cudaSuccess) return err;
 
-  const QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
+  QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
+  // rows are pruned only while the estimate stays internal: a caller's est_out gets every value
+  qp.prune = (qstate && !est_out && can_prune(r, c)) ? 1 : 0;
+  qp.qstate = qstate;
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
-  return select_from_keys(w, est, qp.vec, 0x7FFFFFFFu, d, k, idx_out, s);
+  if (qp.prune) {
+    using T = RepairTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
+    if ((err = T::table[r - 1](qp, w.hist + 3 * kBins, s)) != cudaSuccess) return err;
+  }
+  return select_from_keys(w, est, qp.vec, 0x7FFFFFFFu, d, k, idx_out, s, qstate);
 }
 
 size_t heavymix_workspace_bytes(int64_t d, int64_t k) {
@@ -1014,7 +1144,7 @@ cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, 
   const int nb = (int)nseg;
   if (qp.vec) launch(k_count<true>, nb, kSegThreads, s, est_out, d, st, blk_gt, blk_eq);
   else launch(k_count<false>, nb, kSegThreads, s, est_out, d, st, blk_gt, blk_eq);
-  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, nseg, st, blk_base, blk_eqx);
+  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, nseg, st, blk_base, blk_eqx, (uint32_t*)nullptr, d, (uint32_t)k);
   if (qp.vec) launch(k_write<true>, nb, kSegThreads, s, est_out, d, st, blk_base, blk_eqx, idx_out, k);
   else launch(k_write<false>, nb, kSegThreads, s, est_out, d, st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();

@@ -256,6 +256,49 @@ def test_topk_large_plateau(gs, H, d, k, nonzero):
         run.close()
 
 
+@pytest.mark.parametrize("r,scale", [(5, 1e-3), (5, 0.97), (5, 30.0), (4, 1e-3), (7, 0.5), (3, 1e-3)])
+def test_pruned_query_matches_full_query(gs, H, r, scale):
+    """Queries whose estimate stays in the workspace skip rows below a prune key taken from the
+    sketch's previous query (same d and k).  After a query on x, the sketch is refilled with
+    scale * x (other noise), and queried again internally: with scale = 1e-3 or 0.5 the prune key
+    lies above the new threshold and the repair pass must restore every pruned estimate; with
+    0.97 or 30 pruning is safe.  Either way the selection equals the full query's exactly, every
+    selected estimate is exact, and every pruned (-0.0) one is below the k-th largest |est|."""
+    d, c, k, seed = 1_000_003, 1 << 14, 1000, 40 + r
+    rng = np.random.default_rng(seed)
+    sk = gs.gs_sketch_create(r, c, seed, 1, 0)
+    try:
+        ws = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        est_int = ws[: 4 * d].view(torch.float32)   # the query keeps its estimate at the workspace start
+        idx = torch.empty(k, dtype=torch.int64, device="cuda")
+        idx_full = torch.empty(k, dtype=torch.int64, device="cuda")
+        est_full = torch.empty(d, dtype=torch.float32, device="cuda")
+        for t, sc in enumerate([1.0, scale, scale]):
+            x = (rng.standard_normal(d) * 1e-2).astype(np.float32)
+            x[rng.choice(d, 3000, replace=False)] *= 40
+            x = (x * np.float32(sc)).astype(np.float32)
+            gs.gs_sketch_zero(sk)
+            gs.gs_sketch_insert(sk, 0, _dev(x), d)
+            gs.gs_sketch_merge_tree(sk, 1)
+            gs.gs_query_topk(sk, d, k, idx, None, ws)          # internal estimate: may prune
+            torch.cuda.synchronize()
+            got, e_int = H.host(idx).copy(), H.host(est_int).copy()
+            gs.gs_query_topk(sk, d, k, idx_full, est_full, ws)  # caller's estimate: every row
+            torch.cuda.synchronize()
+            want, e = H.host(idx_full), H.host(est_full)
+            assert np.array_equal(got, want), f"query {t}: selections differ"
+            H.check_selection_exact(got, e, k)
+            pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
+            exact = e_int.view(np.uint32) == e.view(np.uint32)
+            assert np.all(pruned | exact)
+            tau = np.sort(np.abs(e))[-k]
+            assert np.all(np.abs(e[pruned]) < tau) and not pruned[got].any()
+            if t == 0:
+                assert not pruned.any()                         # no record yet: nothing pruned
+    finally:
+        gs.gs_sketch_destroy(sk)
+
+
 def test_topk_all_ties_and_zeros(gs, H):
     d, r, c, k = 50_000, 5, 256, 1234
     run = H.new_run(1, d, r, c, k, 1)
