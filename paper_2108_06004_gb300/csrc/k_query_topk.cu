@@ -924,8 +924,11 @@ struct RepairTable {
 template <int... Rs>
 constexpr RepairLauncher RepairTable<Rs...>::table[sizeof...(Rs)];
 
-// Pruning applies on the fast path (c a power of two) with at least three rows.
-bool can_prune(int r, uint32_t c) { return is_pow2(c) && r >= 3 && r <= GS_MAX_ROWS; }
+// Pruning applies on the fast path (c a power of two) with at least three rows, and from
+// 2^22 coordinates up: below that the query takes a few tens of microseconds and the repair
+// kernel's launch costs more than the skipped rows save (measured on the 2^20 workload).
+constexpr int64_t kPruneMinDim = int64_t(1) << 22;
+bool can_prune(int r, uint32_t c, int64_t d) { return is_pow2(c) && r >= 3 && r <= GS_MAX_ROWS && d >= kPruneMinDim; }
 
 cudaError_t launch_query(const QueryParams& p, cudaStream_t s) {
   using T = QueryTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
@@ -1041,7 +1044,7 @@ cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, u
 
   QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
   // rows are pruned only while the estimate stays internal: a caller's est_out gets every value
-  qp.prune = (qstate && !est_out && can_prune(r, c)) ? 1 : 0;
+  qp.prune = (qstate && !est_out && can_prune(r, c, d)) ? 1 : 0;
   qp.qstate = qstate;
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   if (qp.prune) {

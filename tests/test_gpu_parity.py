@@ -264,7 +264,7 @@ def test_pruned_query_matches_full_query(gs, H, r, scale):
     lies above the new threshold and the repair pass must restore every pruned estimate; with
     0.97 or 30 pruning is safe.  Either way the selection equals the full query's exactly, every
     selected estimate is exact, and every pruned (-0.0) one is below the k-th largest |est|."""
-    d, c, k, seed = 1_000_003, 1 << 14, 1000, 40 + r
+    d, c, k, seed = 4_200_007, 1 << 16, 4000, 40 + r      # pruning applies from d = 2^22
     rng = np.random.default_rng(seed)
     sk = gs.gs_sketch_create(r, c, seed, 1, 0)
     try:
@@ -275,7 +275,7 @@ def test_pruned_query_matches_full_query(gs, H, r, scale):
         est_full = torch.empty(d, dtype=torch.float32, device="cuda")
         for t, sc in enumerate([1.0, scale, scale]):
             x = (rng.standard_normal(d) * 1e-2).astype(np.float32)
-            x[rng.choice(d, 3000, replace=False)] *= 40
+            x[rng.choice(d, 12_000, replace=False)] *= 40
             x = (x * np.float32(sc)).astype(np.float32)
             gs.gs_sketch_zero(sk)
             gs.gs_sketch_insert(sk, 0, _dev(x), d)
@@ -295,6 +295,30 @@ def test_pruned_query_matches_full_query(gs, H, r, scale):
             assert np.all(np.abs(e[pruned]) < tau) and not pruned[got].any()
             if t == 0:
                 assert not pruned.any()                         # no record yet: nothing pruned
+            if t == 2:
+                assert pruned.mean() > 0.3                      # same scale as the query before
+    finally:
+        gs.gs_sketch_destroy(sk)
+
+
+def test_no_pruning_below_4m_coordinates(gs, H):
+    """Under 2^22 coordinates a query reads every row: its internal estimate equals the full one."""
+    d, r, c, k = (1 << 22) - 1, 5, 1 << 14, 500
+    rng = np.random.default_rng(8)
+    sk = gs.gs_sketch_create(r, c, 8, 1, 0)
+    try:
+        gs.gs_sketch_insert(sk, 0, _dev((rng.standard_normal(d) * 1e-2).astype(np.float32)), d)
+        gs.gs_sketch_merge_tree(sk, 1)
+        ws = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        idx = torch.empty(k, dtype=torch.int64, device="cuda")
+        est = torch.empty(d, dtype=torch.float32, device="cuda")
+        for _ in range(2):
+            gs.gs_query_topk(sk, d, k, idx, None, ws)
+        torch.cuda.synchronize()
+        e_int = H.host(ws[: 4 * d].view(torch.float32)).copy()
+        gs.gs_query_topk(sk, d, k, idx, est, ws)
+        torch.cuda.synchronize()
+        assert np.array_equal(e_int.view(np.uint32), H.host(est).view(np.uint32))
     finally:
         gs.gs_sketch_destroy(sk)
 
