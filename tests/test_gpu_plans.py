@@ -222,3 +222,43 @@ def test_step_plan_resnet18_full_size(gs, H):
     finally:
         gs.gs_plan_destroy(plan)
         run.close()
+
+
+def test_step_plan_with_row_pruning(gs, H):
+    """A plan whose estimate stays internal, at a size where the query skips rows (d >= 2^22):
+    after every launch the selection equals a full query of the same merged table, and the
+    gathered values are the exact fp32 sums of the accumulated error vectors."""
+    w = workloads.get_config("resnet18")
+    P, d, r, c, k, seed = 4, 4_500_001, 5, 1 << 16, 4000, 91
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho)
+    gbuf = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+    plan = gs.gs_step_plan_create(run.sketch, run.us, run.es, gbuf, d, w.rho, k, run.idx, run.vals, None,
+                                  workspace=run.ws)
+    ws2 = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+    idx_full = torch.empty(k, dtype=torch.int64, device="cuda")
+    est_full = torch.empty(d, dtype=torch.float32, device="cuda")
+    try:
+        for t in range(4):
+            grads = workloads.make_gradients(w, t, range(P), d=d)
+            for b, g in zip(gbuf, grads):
+                b.copy_(torch.from_numpy(g))
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            gs.gs_plan_launch(plan)
+            gs.gs_query_topk(run.sketch, d, k, idx_full, est_full, ws2)
+            torch.cuda.synchronize()
+            gi = H.host(run.idx)
+            assert np.array_equal(gi, H.host(idx_full)), f"launch {t}: selection differs from the full query"
+            H.check_selection_exact(gi, H.host(est_full), k)
+            e_int = H.host(run.ws[: 4 * d].view(torch.float32))   # the plan's internal estimate
+            pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
+            if t >= 1:
+                assert pruned.mean() > 0.1, "rows were not skipped"
+            es_pre = [oracle.accumulate(u0, e0, g, w.rho)[1] for u0, e0, g in zip(us0, es0, grads)]
+            ref = np.zeros(k, np.float32)
+            for e in es_pre:
+                ref = (ref + e[gi]).astype(np.float32)
+            assert np.array_equal(H.host(run.vals).view(np.uint32), ref.view(np.uint32))
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()
