@@ -197,6 +197,7 @@ def oracle_tie_check(gi, res, k, d):
     (8, 65_536, 4, 4096, 200, 3, 8),
     (6, 31_337, 3, 1500, 100, 3, 2),
     (1, 4_099, 7, 256, 1, 2, 0),
+    (4, 4_200_001, 5, 1 << 16, 4000, 3, 0),   # from 2^22 coordinates the query skips rows
 ])
 def test_sketched_state_steps(gs, P, d, r, c, k, steps, gw):
     _run_steps(gs, P, d, r, c, k, steps, rho=0.9, lr=0.05, seed=d % 977 + P, group_width=gw)
