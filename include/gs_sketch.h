@@ -168,7 +168,11 @@ gs_status gs_query_heavymix_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * (Alg. 2 step 3): those with the smallest xi_i = (i-th splitmix64 output of fill_seed) >> 33,
  * i counted from 0, ties to the smaller index.  idx_out (int64[k]) is ascending; est_out
  * (fp32[d]) and l2sq_out (one device double) may be NULL.  workspace must hold
- * gs_query_heavymix_workspace_size(d, k) bytes, 256-byte aligned. */
+ * gs_query_heavymix_workspace_size(d, k) bytes, 256-byte aligned.
+ * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, a coordinate whose first
+ * r/2 + 1 cells all lie below sqrt(l2sq / k) skips its other rows (its est^2 is below the
+ * threshold, so it can only enter through the fill) and its estimate is left at -0.0 in the
+ * workspace; idx_out is the same as without skipping. */
 gs_status gs_query_heavymix(const gs_sketch* sketch, int64_t d, int64_t k, uint64_t fill_seed,
                             int64_t* idx_out, float* est_out, double* l2sq_out, void* workspace,
                             size_t workspace_bytes, gs_stream stream);

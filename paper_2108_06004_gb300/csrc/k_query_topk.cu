@@ -191,6 +191,7 @@ struct QueryParams {
   int32_t hist_on;    // build the level-1 histogram of |est| keys and pick
   int32_t prune;      // skip rows below the prune key (estimate internal to the workspace)
   uint32_t* qstate;   // the sketch's record of its last query: d (two words), k, tau key
+  const double* theta;  // HEAVYMIX: the threshold l2sq / k on est^2 (prunes below its root)
   HashCoeffs h;
 };
 
@@ -205,6 +206,15 @@ constexpr uint32_t kPrunedBits = 0x80000000u;  // -0.0f: the stored estimate of 
 
 __device__ __forceinline__ uint32_t prune_key_of(const QueryParams& prm) {
   if (!prm.prune) return 0u;
+  if (prm.theta) {
+    // HEAVYMIX: a coordinate with |est| < f, f^2 <= theta, lies outside H, and only its index
+    // enters the selection (through the random fill), so no repair is ever needed
+    const double th = __ldcg(prm.theta);
+    if (!(th > 0.0) || th > 1e300) return 0u;
+    float f = __double2float_rd(sqrt(th));
+    if ((double)f * (double)f > th) f = nextafterf(f, 0.f);  // the product is exact in double
+    return key_of(f) & ~((1u << kL1Shift) - 1u);
+  }
   const uint32_t dl = __ldcg(&prm.qstate[0]), dh = __ldcg(&prm.qstate[1]);
   const uint32_t kk = __ldcg(&prm.qstate[2]), tk = __ldcg(&prm.qstate[3]);
   if (dl != (uint32_t)prm.d || dh != (uint32_t)((uint64_t)prm.d >> 32) || kk != prm.k) return 0u;
@@ -953,6 +963,7 @@ QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, u
   qp.hist_on = 1;
   qp.prune = 0;
   qp.qstate = nullptr;
+  qp.theta = nullptr;
   qp.h = h;
   return qp;
 }
@@ -1071,13 +1082,16 @@ cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int 
   if (err == cudaSuccess) err = cudaMemsetAsync(sumsq, 0, 256, s);
   if (err != cudaSuccess) return err;
 
-  QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
-  qp.hist_on = 0;
-  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
+  // the threshold first (it reads only the table), so that the query can skip rows below it
   const int gx = (int)(((int64_t)c + kBlock - 1) / kBlock < 4 * device_info().sms ? ((int64_t)c + kBlock - 1) / kBlock
                                                                                   : 4 * device_info().sms);
   launch(k_row_sumsq, dim3(gx, r), kBlock, s, merged, c, sumsq);
   launch(k_heavy_theta, 1, 32, s, sumsq, r, k, theta, l2sq_out);
+  QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
+  qp.hist_on = 0;
+  qp.prune = (!est_out && can_prune(r, c, d)) ? 1 : 0;
+  qp.theta = theta;
+  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   launch(k_heavy_keys, persistent_grid(k_heavy_keys, d, kBlock), kBlock, s, est, d, theta, fill_seed, keys, w.hist,
                                                                            w.st, (uint32_t)k);
   return select_from_keys(w, reinterpret_cast<const float*>(keys), 1, 0xFFFFFFFFu, d, k, idx_out, s);

@@ -553,6 +553,41 @@ def test_train_steps(gs, H):
 
 # ---- HEAVYMIX (Alg. 2 as printed) ----------------------------------------------------------
 
+@pytest.mark.parametrize("r,k,spikes", [(5, 4000, 800), (4, 3000, 5000), (7, 20000, 300)])
+def test_heavymix_pruned_matches_full(gs, H, r, k, spikes):
+    """From 2^22 coordinates a HEAVYMIX query with an internal estimate skips the rows of
+    coordinates whose first r/2 + 1 cells bound est^2 below l2sq / k: they lie outside H and
+    enter the selection only through the random fill.  The selection equals the query that
+    returns every estimate, and rows were in fact skipped."""
+    d, c, seed, fill_seed = 4_200_007, 1 << 16, 17 + r, 2**62 + 3
+    rng = np.random.default_rng(seed)
+    x = (rng.standard_normal(d) * 1e-3).astype(np.float32)
+    x[rng.choice(d, spikes, replace=False)] *= np.float32(60.0)
+    sk = gs.gs_sketch_create(r, c, seed, 1, 0)
+    try:
+        gs.gs_sketch_insert(sk, 0, _dev(x), d)
+        gs.gs_sketch_merge_tree(sk, 1)
+        ws = torch.empty(gs.gs_query_heavymix_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        l2 = torch.empty(2, dtype=torch.float64, device="cuda")
+        idx_full = torch.empty(k, dtype=torch.int64, device="cuda")
+        idx = torch.empty(k, dtype=torch.int64, device="cuda")
+        est = torch.empty(d, dtype=torch.float32, device="cuda")
+        gs.gs_query_heavymix(sk, d, k, fill_seed, idx_full, est, l2[0:1], ws)
+        gs.gs_query_heavymix(sk, d, k, fill_seed, idx, None, l2[1:2], ws)
+        torch.cuda.synchronize()
+        e_int = H.host(ws[: 4 * d].view(torch.float32))
+        assert np.array_equal(H.host(idx), H.host(idx_full))
+        l2h = H.host(l2)
+        assert abs(l2h[0] - l2h[1]) <= 1e-12 * l2h[0]   # fp64 atomic sums: order varies
+        assert np.array_equal(H.host(idx_full), oracle.heavymix_select(H.host(est), float(l2h[0]), k, fill_seed))
+        pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
+        assert pruned.mean() > 0.2, "rows were not skipped"
+        e = H.host(est).astype(np.float64)
+        assert np.all(e[pruned] ** 2 < l2h[0] / k)
+    finally:
+        gs.gs_sketch_destroy(sk)
+
+
 @pytest.mark.parametrize("d,r,c,k,spikes,scale", [(400_003, 5, 1 << 12, 300, 40, 50.0),
                                                   (400_003, 5, 1 << 12, 5, 40, 50.0),
                                                   (250_001, 4, 3001, 2000, 10, 20.0),
