@@ -472,6 +472,14 @@ def _oracle_sample_step(w, t, d_s, k_s, coeffs, us, es):
     return dt, res
 
 
+def host_cores() -> int:
+    """Host cores this process may run on."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        return os.cpu_count() or 1
+
+
 def cpu_baseline(w, steps=1, d_s=CPU_SAMPLE_D):
     """The oracle, as it stands, on the first d_s coordinates of each worker's gradient
     (same P, r, c and rho; k scaled with d); the same unit as the metric."""
@@ -486,7 +494,8 @@ def cpu_baseline(w, steps=1, d_s=CPU_SAMPLE_D):
         dt, res = _oracle_sample_step(w, t, d_s, k_s, coeffs, us, es)
         total += dt
         us, es = res.us, res.es
-    return {"value": w.P * d_s * steps / total, "unit": UNIT, "cores": 1, "kind": "oracle",
+    return {"value": w.P * d_s * steps / total, "unit": UNIT, "cores": 1, "cores_available": host_cores(),
+            "processes": 1, "kind": "oracle",
             "sample": f"{steps} step(s) of the oracle on the first {d_s} coordinates of each of the {w.P} "
                       f"workers (r={w.r}, c={w.c}, k={k_s}), numpy single-threaded"}
 
@@ -522,7 +531,8 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total * 1e3 / args.steps, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "d": w.d, "P": w.P, "r": w.r, "c": w.c, "k": w.k, "rho": w.rho},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "cores_available": host_cores(), "processes": 1,
+                         "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
