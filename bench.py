@@ -440,7 +440,9 @@ def run_ours(args):
             gs.gs_sketch_destroy(extra)
     # insert (one per group and row pass), merge, query + selection (7; HEAVYMIX 10), then
     # the gather (sketched state: cell accumulate, take, query_at, two sparse inserts, update)
-    launches_per_step = groups * passes + 1 + (10 if variant == "heavymix" else 7) + \
+    # the top-k query adds its repair check where it prunes rows (d >= 2^22, r >= 3, c a power of two)
+    prunes = variant != "heavymix" and d >= (1 << 22) and r >= 3 and (c & (c - 1)) == 0
+    launches_per_step = groups * passes + 1 + (10 if variant == "heavymix" else 7) + (1 if prunes else 0) + \
         (6 if variant == "sketched_state" else 1)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
