@@ -262,3 +262,43 @@ def test_step_plan_with_row_pruning(gs, H):
     finally:
         gs.gs_plan_destroy(plan)
         run.close()
+
+
+def test_step_plan_repairs_a_stale_prune_key(gs, H):
+    """Inside a plan the repair of a too-high prune key runs as a graph node: after a launch on
+    normal gradients, momentum and error are cleared and the next launch gets gradients 1000
+    times smaller, so the key from the first launch lies far above the new threshold."""
+    w = workloads.get_config("resnet18")
+    P, d, r, c, k, seed = 2, 4_300_001, 5, 1 << 16, 3000, 93
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho)
+    gbuf = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+    plan = gs.gs_step_plan_create(run.sketch, run.us, run.es, gbuf, d, w.rho, k, run.idx, run.vals, None,
+                                  workspace=run.ws)
+    ws2 = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+    idx_full = torch.empty(k, dtype=torch.int64, device="cuda")
+    est_full = torch.empty(d, dtype=torch.float32, device="cuda")
+    try:
+        for t, scale in enumerate([1.0, 1e-3]):
+            grads = [(g * np.float32(scale)).astype(np.float32) for g in workloads.make_gradients(w, t, range(P), d=d)]
+            for b, g in zip(gbuf, grads):
+                b.copy_(torch.from_numpy(g))
+            for u, e in zip(run.us, run.es):
+                u.zero_()
+                e.zero_()
+            gs.gs_plan_launch(plan)
+            torch.cuda.synchronize()
+            gi = H.host(run.idx).copy()
+            e_int = H.host(run.ws[: 4 * d].view(torch.float32))
+            # the record now holds this launch's threshold: query the same table in full
+            gs.gs_query_topk(run.sketch, d, k, idx_full, est_full, ws2)
+            torch.cuda.synchronize()
+            assert np.array_equal(gi, H.host(idx_full)), f"launch {t}: selection differs from the full query"
+            if t == 1:   # repaired: every estimate is the full one
+                assert np.array_equal(e_int.view(np.uint32), H.host(est_full).view(np.uint32))
+            ref = np.zeros(k, np.float32)
+            for g in grads:   # from cleared state, e = u = g
+                ref = (ref + g[gi]).astype(np.float32)
+            assert np.array_equal(H.host(run.vals).view(np.uint32), ref.view(np.uint32))
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()
