@@ -30,7 +30,8 @@
  *     the vectorised path (results are identical either way).
  *   - Sizes: 1 <= r <= GS_MAX_ROWS, 1 <= c <= GS_MAX_COLS, 1 <= d <= GS_MAX_DIM,
  *     1 <= k <= d, 1 <= P <= GS_MAX_WORKERS.  Vector values must be finite.
- *   - No call waits on the device for a flag; nothing spins.
+ *   - No call waits on the device for a flag; nothing spins.  Kernels launch with
+ *     programmatic stream serialization and wait in hardware for the grid before them.
  */
 #ifndef GS_SKETCH_H
 #define GS_SKETCH_H
@@ -69,8 +70,8 @@ typedef struct gs_plan gs_plan;     /* opaque: one step captured into a CUDA gra
  * cell are adjacent and are updated by 16-byte vector reductions (G = group_width/4 lanes
  * together write a whole cell in one instruction); group_width 0 lets the library choose
  * (up to 16, no wider than the worker count rounded up to a power of two; 16 only when the
- * whole group table fits a 64 MiB L2 budget, and halved while one table row exceeds it).  The fused insert updates as many rows per pass
- * as fit that budget.
+ * whole group table fits 48 MiB of L2, and halved while one table row exceeds 64 MiB).  The
+ * fused insert updates as many rows per pass as fit 48 MiB, and at least one.
  * On success *out owns device memory released by gs_sketch_destroy.
  * Errors: GS_ERR_INVALID_ARG (sizes, group_width not in {0,1,2,4,8,16}, out NULL),
  *         GS_ERR_OOM (allocation failed), GS_ERR_CUDA.  Synchronous. */
