@@ -148,11 +148,13 @@ gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * and two d-bit bitmaps).
  * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, the query may skip rows: a
  * coordinate whose first r/2 + 1 cells are all below a threshold cannot be selected (they
- * bound the median), and its estimate is left at -0.0 in the workspace.  The threshold comes
- * from this sketch's previous top-k query with the same d and k (16 bytes the sketch keeps),
- * and when it turns out too high the skipped estimates are recomputed.  idx_out is exactly the
- * same as without skipping; only the time differs.  Queries of one sketch on different
- * streams may interleave their record of the threshold; that only changes the time.
+ * bound the median), and its estimate is left at -0.0 in the workspace.  The threshold is
+ * taken by the same call before the main pass, from the full estimate of a fixed sample (the
+ * first four coordinates of every 256): the level-1 bin edge below a rank of the sample chosen
+ * so that the threshold lies under the k-th largest |est| except with negligible probability.
+ * When it does not, the skipped estimates are recomputed.  idx_out is exactly the same as
+ * without skipping; only the time differs.  The threshold lives in the workspace, so queries
+ * on different streams with different workspaces are independent.
  * gs_step, gs_train_step, gs_step_host and gs_sketched_state_step query the same way. */
 gs_status gs_query_topk(const gs_sketch* sketch, int64_t d, int64_t k, int64_t* idx_out,
                         float* est_out, void* workspace, size_t workspace_bytes,

@@ -16,7 +16,6 @@ struct gs_sketch {
   gs::HashCoeffs h;
   float* tables;  // groups * r*c*W
   float* merged;  // r*c
-  uint32_t* qstate;  // last top-k query of the merged table: d (two words), k, threshold key
   int device;
 };
 
@@ -239,7 +238,7 @@ gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float
   mp.group_stride = (int64_t)sk->r * sk->c * sk->W;
   mp.P = sk->workers;
   if ((err = gs::launch_merge(mp, sk->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
-  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, s, sk->qstate)) !=
+  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, s)) !=
       cudaSuccess)
     return cuda_fail(err, "query/top-k launch");
   gs::GatherParams gp;
@@ -321,7 +320,7 @@ gs_status sketched_state_impl(gs_sketch* workers, gs_sketch* momentum, gs_sketch
     return cuda_fail(err, "sketch accumulate launch");
   // top-k of the estimate from E; delta = that estimate at the selected coordinates
   if ((err = gs::launch_query_topk(error->merged, error->h, error->r, (uint32_t)error->c, d, k, idx, nullptr,
-                                   ws, s, error->qstate)) != cudaSuccess)
+                                   ws, s)) != cudaSuccess)
     return cuda_fail(err, "query/top-k launch");
   const float* est = static_cast<const float*>(ws);  // the query keeps est at the ws start
   if ((err = gs::launch_take(est, d, idx, k, vals, s)) != cudaSuccess) return cuda_fail(err, "take launch");
@@ -575,7 +574,7 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   const int W = group_width ? group_width : choose_group_width(r, c, workers);
   const int groups = (workers + W - 1) / W;
   const size_t table_floats = (size_t)groups * r * c * W;
-  const size_t bytes = (table_floats + (size_t)r * c) * sizeof(float) + 16;  // + qstate
+  const size_t bytes = (table_floats + (size_t)r * c) * sizeof(float);
   float* mem = nullptr;
   e = cudaMalloc(&mem, bytes);
   if (e != cudaSuccess) {
@@ -599,7 +598,6 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   derive_coefficients(r, seed, sk->h);
   sk->tables = mem;
   sk->merged = mem + table_floats;
-  sk->qstate = reinterpret_cast<uint32_t*>(sk->merged + (size_t)r * c);
   sk->device = dev;
   *out = sk;
   return ok();
@@ -734,7 +732,7 @@ gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_
   if (workspace_bytes < gs::query_topk_workspace_bytes(d, k))
     return fail(GS_ERR_INVALID_ARG, "workspace too small: need " + std::to_string(gs::query_topk_workspace_bytes(d, k)));
   cudaError_t e = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx_out, est_out, workspace,
-                                        as_stream(stream), sk->qstate);
+                                        as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "query/top-k launch");
   return GS_OK;
 }
@@ -767,6 +765,7 @@ gs_status gs_query_heavymix(const gs_sketch* sk, int64_t d, int64_t k, uint64_t 
 
 gs_status gs_query_topk_noalloc(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_out, float* est_out,
                                 gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   GS_TRY(check_d(d));
   if (d > GS_NOALLOC_MAX_DIM)
@@ -781,6 +780,7 @@ gs_status gs_query_topk_noalloc(const gs_sketch* sk, int64_t d, int64_t k, int64
                                                 as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "query/top-k (no-allocation variant)");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_gather_and_zero(float* const* momentum, float* const* error, int32_t P, int64_t d, const int64_t* idx,

@@ -132,11 +132,9 @@ cudaError_t launch_query_at(const float* T, const HashCoeffs& h, int r, uint32_t
 cudaError_t launch_add_sparse(float* T, const HashCoeffs& h, int r, uint32_t c, const int64_t* idx, const float* vals,
                               int64_t k, float scale, cudaStream_t s);
 cudaError_t launch_take(const float* src, int64_t n, const int64_t* idx, int64_t k, float* out, cudaStream_t s);
-// qstate (nullable): the sketch's record of its last top-k query (4 words), read for the prune
-// key and rewritten with this query's threshold.
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, cudaStream_t s, uint32_t* qstate = nullptr);
+                              void* workspace, cudaStream_t s);
 // HEAVYMIX selection (Alg. 2 as printed) from the merged table; l2sq_out (device double,
 // nullable) receives the sketch's estimate of ||g||^2.
 size_t heavymix_workspace_bytes(int64_t d, int64_t k);

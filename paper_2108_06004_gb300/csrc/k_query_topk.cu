@@ -11,10 +11,12 @@
 // smallest index.  Output indices are ascending.
 //
 // With a caller workspace (gs_query_topk):
+//   k_qsample     (only where rows are pruned) the full estimate of a fixed strided sample of
+//                 coordinates, its level-1 histogram, and a prune key from it: a lower bound
+//                 on the k-th largest |est| of this query, rounded down to a bin edge
 //   k_query       est_i for every i (fp32) + level-1 histogram + pick; when the estimate stays
 //                 in the workspace, a coordinate whose first r/2 + 1 rows all lie below the
-//                 prune key (from the sketch's previous query) skips its other rows and stores
-//                 -0.0 (see below)
+//                 prune key skips its other rows and stores -0.0 (see below)
 //   k_repair      runs only if the level-1 pick fell below the prune key: recomputes every
 //                 -0.0 estimate in full, rebuilds the level-1 histogram and picks again
 //   k_cand        one pass over est: keys above the picked level-1 bin are selected for
@@ -27,7 +29,10 @@
 //   k_bm_write    every block writes its selected indices at their final positions
 // With the fixed scratch (gs_query_topk_noalloc), which cannot hold candidate lists, the
 // levels 2 and 3 and the final selection read est in full passes (k_hist, k_count, k_write).
+#include <cmath>
 #include <mutex>
+
+#include <cuda.h>
 
 #include "gs_common.cuh"
 
@@ -51,8 +56,10 @@ struct SelectState {
   uint32_t found;    // bit l set when level l found its bin
   uint32_t ncand;    // candidates appended by k_cand
   uint32_t done[3];  // CTAs finished per level (for the last-CTA pick)
-  uint32_t prune_key;  // the key below which k_query skipped rows (0: none)
+  uint32_t prune_key;  // the key below which k_query skips rows (0: none); written once per
+                       // query, before k_query, by k_qsample or k_heavy_theta
   uint32_t done_r;     // CTAs finished in k_repair
+  uint32_t done_s;     // CTAs finished in k_qsample
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -189,37 +196,23 @@ struct QueryParams {
   uint32_t c, cmask;
   int32_t vec;        // est 16-byte aligned
   int32_t hist_on;    // build the level-1 histogram of |est| keys and pick
-  int32_t prune;      // skip rows below the prune key (estimate internal to the workspace)
-  uint32_t* qstate;   // the sketch's record of its last query: d (two words), k, tau key
-  const double* theta;  // HEAVYMIX: the threshold l2sq / k on est^2 (prunes below its root)
+  int32_t prune;      // skip rows below st->prune_key (estimate internal to the workspace)
   HashCoeffs h;
 };
 
 // Row pruning.  The median of r values lies between the least and the largest of any
 // r/2 + 1 of them (for even r both middle values do, and so does their fp32 mean).  So a
 // coordinate whose first r/2 + 1 signed cells all have |v| < t has |est| < t and cannot be
-// among the top k when t is at most the k-th largest |est|.  The prune key is 0.9 times the
-// k-th largest key of the sketch's previous query with the same d and k, rounded down to a
-// level-1 bin edge: whether it was safe is then exactly whether the level-1 pick lands in
-// that bin or above, which k_repair checks.
+// among the top k when t is at most the k-th largest |est|.  The prune key t is computed by
+// this query itself before k_query runs (k_qsample: from the full estimate of a strided
+// sample of coordinates; HEAVYMIX: from its threshold) and kept in the query's own selection
+// state, so every CTA of k_query and k_repair reads the same value.  It is a level-1 bin
+// edge: whether it was safe is then exactly whether the level-1 pick lands in its bin or
+// above, which k_repair checks.
 constexpr uint32_t kPrunedBits = 0x80000000u;  // -0.0f: the stored estimate of a pruned coordinate
 
 __device__ __forceinline__ uint32_t prune_key_of(const QueryParams& prm) {
-  if (!prm.prune) return 0u;
-  if (prm.theta) {
-    // HEAVYMIX: a coordinate with |est| < f, f^2 <= theta, lies outside H, and only its index
-    // enters the selection (through the random fill), so no repair is ever needed
-    const double th = __ldcg(prm.theta);
-    if (!(th > 0.0) || th > 1e300) return 0u;
-    float f = __double2float_rd(sqrt(th));
-    if ((double)f * (double)f > th) f = nextafterf(f, 0.f);  // the product is exact in double
-    return key_of(f) & ~((1u << kL1Shift) - 1u);
-  }
-  const uint32_t dl = __ldcg(&prm.qstate[0]), dh = __ldcg(&prm.qstate[1]);
-  const uint32_t kk = __ldcg(&prm.qstate[2]), tk = __ldcg(&prm.qstate[3]);
-  if (dl != (uint32_t)prm.d || dh != (uint32_t)((uint64_t)prm.d >> 32) || kk != prm.k) return 0u;
-  if (tk == 0u || tk >= 0x7F800000u) return 0u;
-  return key_of(0.9f * __uint_as_float(tk)) & ~((1u << kL1Shift) - 1u);
+  return prm.prune ? __ldcg(&prm.st->prune_key) : 0u;
 }
 
 __device__ __forceinline__ void store_est(const QueryParams& prm, int64_t i0, int tmax,
@@ -245,7 +238,6 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int lane = threadIdx.x & 31;
   const uint32_t pk = prune_key_of(prm);
-  if (prm.prune && blockIdx.x == 0 && threadIdx.x == 0) prm.st->prune_key = pk;
   constexpr int kF = R / 2 + 1;  // rows that bound the median
   for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += stride) {
     const int64_t q = q0 + lane;
@@ -345,6 +337,79 @@ __global__ void __launch_bounds__(kBlock) k_repair(const __grid_constant__ Query
   }
   hist_flush(sh, hist_r, kBins);
   last_block_pick(hist_r, 11, prm.st, 0, prm.k, &prm.st->done_r);
+}
+
+// The prune key of this query, from a fixed strided sample: the first four coordinates of
+// every kSampleQuads * 4 (all rows, full median).  The last CTA finds the level-1 bin holding
+// the j_target-th largest sampled key and stores its lower edge as st->prune_key (0, i.e. no
+// pruning, when that is bin 0 or the sample holds fewer keys).  j_target is set on the host
+// well above the sample's expected share of the top k, so that the key lies below the k-th
+// largest |est| of the whole estimate except with negligible probability; k_repair makes the
+// result exact in that case as well.
+constexpr int64_t kSampleQuads = 64;
+
+template <int R>
+__global__ void __launch_bounds__(kBlock) k_qsample(const __grid_constant__ QueryParams prm, uint32_t* hist_s,
+                                                    uint32_t j_target) {
+  grid_begin();
+  __shared__ uint32_t sh[kBins];
+  __shared__ uint32_t am_last;
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
+  __syncthreads();
+  const int64_t d = prm.d, nq = (d + 3) / 4, ns = (nq + kSampleQuads - 1) / kSampleQuads;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int lane = threadIdx.x & 31;
+  for (int64_t s0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); s0 < ns; s0 += stride) {
+    const int64_t sq = s0 + lane;
+    const int64_t i0 = sq * kSampleQuads * 4;
+    const int tmax = sq < ns ? (d - i0 < 4 ? (int)(d - i0) : 4) : 0;
+    float m[4] = {0.f, 0.f, 0.f, 0.f};
+    if (tmax > 0) {
+      float v[4][R];
+#pragma unroll
+      for (int j = 0; j < R; ++j) {
+        uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+        uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
+        const float* row = prm.T + (size_t)j * prm.c;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          v[t][j] = 0.f;
+          if (t < tmax) {
+            v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
+            x = step61(x, prm.h.a[j]);
+            y = step61(y, prm.h.a2[j]);
+          }
+        }
+      }
+#pragma unroll
+      for (int t = 0; t < 4; ++t) m[t] = median_of<R>(v[t]);
+    }
+#pragma unroll
+    for (int t = 0; t < 4; ++t) hist_add(sh, t < tmax ? (key_of(m[t]) >> kL1Shift) : kNone);
+  }
+  hist_flush(sh, hist_s, kBins);
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) am_last = (atomicAdd(&prm.st->done_s, 1u) == gridDim.x - 1) ? 1u : 0u;
+  __syncthreads();
+  if (!am_last) return;
+  __threadfence();
+  const int per = (kBins + blockDim.x - 1) / blockDim.x;
+  const int r0 = threadIdx.x * per;  // positions counted from the top bin
+  uint32_t local = 0;
+  for (int t = 0; t < per; ++t) {
+    if (r0 + t < kBins) local += __ldcg(&hist_s[kBins - 1 - (r0 + t)]);
+  }
+  uint32_t total;
+  uint32_t cum = block_excl_scan(local, &total);
+  for (int t = 0; t < per; ++t) {
+    const int rp = r0 + t;
+    if (rp >= kBins) break;
+    const int bin = kBins - 1 - rp;
+    const uint32_t cnt = __ldcg(&hist_s[bin]);
+    if (cum < j_target && cum + cnt >= j_target) prm.st->prune_key = bin > 0 ? (uint32_t)bin << kL1Shift : 0u;
+    cum += cnt;
+  }
 }
 
 // General path: any r <= 16 and any c (bucket by 64-bit remainder).
@@ -557,16 +622,9 @@ __global__ void __launch_bounds__(kBmThreads) k_bm_count(const uint32_t* __restr
 __global__ void __launch_bounds__(kScanThreads) k_scan(const uint32_t* __restrict__ blk_gt,
                                                        const uint32_t* __restrict__ blk_eq, int64_t nblk,
                                                        const SelectState* st, uint32_t* blk_base,
-                                                       uint32_t* blk_eqx, uint32_t* qstate, int64_t d,
-                                                       uint32_t k) {
+                                                       uint32_t* blk_eqx) {
   grid_begin();
   const uint32_t need_eq = __ldcg(&st->need_eq);
-  if (qstate && threadIdx.x == 0) {  // the sketch's record of this query, for the next one's prune key
-    qstate[0] = (uint32_t)d;
-    qstate[1] = (uint32_t)((uint64_t)d >> 32);
-    qstate[2] = k;
-    qstate[3] = __ldcg(&st->tau);
-  }
   uint32_t carry_gt = 0, carry_eq = 0;
   for (int64_t c0 = 0; c0 < nblk; c0 += blockDim.x) {
     const int64_t b = c0 + threadIdx.x;
@@ -829,8 +887,11 @@ __global__ void __launch_bounds__(kBlock) k_row_sumsq(const float* __restrict__ 
 
 // l2sq = median over rows of the row sums of squares (the sketch's estimate of ||g||^2);
 // theta = l2sq / k, the threshold of H.
+// With `prune`, also the prune key of the query that follows: a coordinate with |est| < f,
+// f^2 <= theta, lies outside H, and only its index enters the selection (through the random
+// fill), so no repair is ever needed.
 __global__ void k_heavy_theta(const double* __restrict__ sumsq, int r, int64_t k, double* theta,
-                              double* l2sq_out) {
+                              double* l2sq_out, SelectState* st, int prune) {
   grid_begin();
   if (blockIdx.x != 0 || threadIdx.x != 0) return;
   double v[GS_MAX_ROWS];
@@ -845,8 +906,14 @@ __global__ void k_heavy_theta(const double* __restrict__ sumsq, int r, int64_t k
     v[b + 1] = t;
   }
   const double m = (r & 1) ? v[r / 2] : 0.5 * (v[r / 2 - 1] + v[r / 2]);
-  theta[0] = m / (double)k;
+  const double th = m / (double)k;
+  theta[0] = th;
   if (l2sq_out) l2sq_out[0] = m;
+  if (prune && th > 0.0 && th <= 1e300) {
+    float f = __double2float_rd(sqrt(th));
+    if ((double)f * (double)f > th) f = nextafterf(f, 0.f);  // the product is exact in double
+    st->prune_key = key_of(f) & ~((1u << kL1Shift) - 1u);
+  }
 }
 
 // The i-th output (i = 0, 1, ...) of the splitmix64 stream seeded with `seed`: the state after
@@ -934,6 +1001,37 @@ struct RepairTable {
 template <int... Rs>
 constexpr RepairLauncher RepairTable<Rs...>::table[sizeof...(Rs)];
 
+template <int R>
+cudaError_t launch_qsample_r(const QueryParams& p, uint32_t* hist_s, uint32_t j_target, cudaStream_t s) {
+  auto kern = k_qsample<R>;
+  const int64_t ns = ((p.d + 3) / 4 + kSampleQuads - 1) / kSampleQuads;
+  launch(kern, persistent_grid(kern, ns, kBlock), kBlock, s, p, hist_s, j_target);
+  return cudaGetLastError();
+}
+
+typedef cudaError_t (*SampleLauncher)(const QueryParams&, uint32_t*, uint32_t, cudaStream_t);
+
+template <int... Rs>
+struct SampleTable {
+  static constexpr SampleLauncher table[sizeof...(Rs)] = {&launch_qsample_r<Rs>...};
+};
+template <int... Rs>
+constexpr SampleLauncher SampleTable<Rs...>::table[sizeof...(Rs)];
+
+// Rank, among the sampled keys, whose level-1 bin gives the prune key.  The sample holds n_s
+// of the d coordinates; the number of them among the k - 1 keys above the k-th largest is
+// at most hypergeometric with mean mu = k n_s / d.  Taking rank mu + 4 sqrt(mu) + 2 puts the
+// sampled key below the k-th largest unless that count exceeds its mean by four standard
+// deviations; for k below that rank it cannot exceed it at all.  0: no usable rank.
+uint32_t sample_rank(int64_t d, int64_t k) {
+  const int64_t ns = ((d + 3) / 4 + kSampleQuads - 1) / kSampleQuads;
+  const int64_t last = (ns - 1) * kSampleQuads * 4;
+  const int64_t n_s = 4 * (ns - 1) + (d - last < 4 ? d - last : 4);
+  const double mu = (double)k * (double)n_s / (double)d;
+  const double j = std::ceil(mu + 4.0 * std::sqrt(mu)) + 2.0;
+  return j <= (double)n_s ? (uint32_t)j : 0u;
+}
+
 // Pruning applies on the fast path (c a power of two) with at least three rows, and from
 // 2^22 coordinates up: below that the query takes a few tens of microseconds and the repair
 // kernel's launch costs more than the skipped rows save (measured on the 2^20 workload).
@@ -962,8 +1060,6 @@ QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, u
   qp.vec = (reinterpret_cast<uintptr_t>(est) & 15u) == 0 ? 1 : 0;
   qp.hist_on = 1;
   qp.prune = 0;
-  qp.qstate = nullptr;
-  qp.theta = nullptr;
   qp.h = h;
   return qp;
 }
@@ -971,7 +1067,7 @@ QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, u
 // Layout of the caller's workspace for the candidate pipeline.
 struct Workspace {
   float* est;         // d
-  uint32_t* hist;     // 4 * kBins: levels 1-3, and level 1 again for k_repair
+  uint32_t* hist;     // 5 * kBins: levels 1-3, level 1 again for k_repair, the sample's level 1
   SelectState* st;
   uint2* cand;        // d (index, key) pairs: room for every coordinate
   uint32_t* gt_bm;    // nbw words
@@ -988,7 +1084,7 @@ Workspace carve(void* base, int64_t d) {
   w.est = reinterpret_cast<float*>(p);
   p += align256((size_t)d * sizeof(float));
   w.hist = reinterpret_cast<uint32_t*>(p);
-  p += align256(4 * kBins * sizeof(uint32_t));
+  p += align256(5 * kBins * sizeof(uint32_t));
   w.st = reinterpret_cast<SelectState*>(p);
   p += align256(sizeof(SelectState));
   w.cand = reinterpret_cast<uint2*>(p);
@@ -1007,7 +1103,7 @@ size_t query_topk_workspace_bytes(int64_t d, int64_t k) {
   (void)k;
   const int64_t nbw = (d + 31) / 32;
   const int64_t nblk = (nbw + kBmWords - 1) / kBmWords;
-  return align256((size_t)d * sizeof(float)) + align256(4 * kBins * sizeof(uint32_t)) +
+  return align256((size_t)d * sizeof(float)) + align256(5 * kBins * sizeof(uint32_t)) +
          align256(sizeof(SelectState)) + align256((size_t)d * sizeof(uint2)) +
          2 * align256((size_t)nbw * sizeof(uint32_t)) + align256((size_t)nblk * 4 * sizeof(uint32_t));
 }
@@ -1016,7 +1112,7 @@ namespace {
 
 // Histograms, state and both bitmaps back to zero.
 cudaError_t clear_selection(const Workspace& w, cudaStream_t s) {
-  cudaError_t err = cudaMemsetAsync(w.hist, 0, 4 * kBins * sizeof(uint32_t), s);
+  cudaError_t err = cudaMemsetAsync(w.hist, 0, 5 * kBins * sizeof(uint32_t), s);
   if (err == cudaSuccess) err = cudaMemsetAsync(w.st, 0, sizeof(SelectState), s);
   // the two bitmaps are adjacent: clear both at once
   if (err == cudaSuccess)
@@ -1026,7 +1122,7 @@ cudaError_t clear_selection(const Workspace& w, cudaStream_t s) {
 
 // Levels 2 and 3 and the ordered output, after the level-1 histogram and pick of `src` keys.
 cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint32_t kmask, int64_t d, int64_t k,
-                             int64_t* idx_out, cudaStream_t s, uint32_t* qstate = nullptr) {
+                             int64_t* idx_out, cudaStream_t s) {
   launch(k_cand, persistent_grid(k_cand, (d + 3) / 4 / kU, kBlock), kBlock, s, src, d, vec, kmask, w.st,
                                                                                  w.hist + kBins, w.cand, w.gt_bm);
   const int small_grid = device_info().sms;
@@ -1038,7 +1134,7 @@ cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint
   uint32_t* blk_eqx = blk_base + w.nblk;
   const int nb = (int)w.nblk;
   launch(k_bm_count, nb, kBmThreads, s, w.gt_bm, w.eq_bm, w.nbw, blk_gt, blk_eq);
-  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx, qstate, d, (uint32_t)k);
+  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, w.nblk, w.st, blk_base, blk_eqx);
   launch(k_bm_write, nb, kBmThreads, s, w.gt_bm, w.eq_bm, w.nbw, w.st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();
 }
@@ -1047,7 +1143,7 @@ cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint
 
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, cudaStream_t s, uint32_t* qstate) {
+                              void* workspace, cudaStream_t s) {
   Workspace w = carve(workspace, d);
   float* est = est_out ? est_out : w.est;
   cudaError_t err = clear_selection(w, s);
@@ -1055,14 +1151,18 @@ cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, u
 
   QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
   // rows are pruned only while the estimate stays internal: a caller's est_out gets every value
-  qp.prune = (qstate && !est_out && can_prune(r, c, d)) ? 1 : 0;
-  qp.qstate = qstate;
+  const uint32_t j_target = sample_rank(d, k);
+  qp.prune = (!est_out && can_prune(r, c, d) && j_target > 0) ? 1 : 0;
+  if (qp.prune) {
+    using T = SampleTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
+    if ((err = T::table[r - 1](qp, w.hist + 4 * kBins, j_target, s)) != cudaSuccess) return err;
+  }
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   if (qp.prune) {
     using T = RepairTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
     if ((err = T::table[r - 1](qp, w.hist + 3 * kBins, s)) != cudaSuccess) return err;
   }
-  return select_from_keys(w, est, qp.vec, 0x7FFFFFFFu, d, k, idx_out, s, qstate);
+  return select_from_keys(w, est, qp.vec, 0x7FFFFFFFu, d, k, idx_out, s);
 }
 
 size_t heavymix_workspace_bytes(int64_t d, int64_t k) {
@@ -1086,11 +1186,11 @@ cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int 
   const int gx = (int)(((int64_t)c + kBlock - 1) / kBlock < 4 * device_info().sms ? ((int64_t)c + kBlock - 1) / kBlock
                                                                                   : 4 * device_info().sms);
   launch(k_row_sumsq, dim3(gx, r), kBlock, s, merged, c, sumsq);
-  launch(k_heavy_theta, 1, 32, s, sumsq, r, k, theta, l2sq_out);
+  const int prune = (!est_out && can_prune(r, c, d)) ? 1 : 0;
+  launch(k_heavy_theta, 1, 32, s, sumsq, r, k, theta, l2sq_out, w.st, prune);
   QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
   qp.hist_on = 0;
-  qp.prune = (!est_out && can_prune(r, c, d)) ? 1 : 0;
-  qp.theta = theta;
+  qp.prune = prune;
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   launch(k_heavy_keys, persistent_grid(k_heavy_keys, d, kBlock), kBlock, s, est, d, theta, fill_seed, keys, w.hist,
                                                                            w.st, (uint32_t)k);
@@ -1112,22 +1212,65 @@ static_assert(sizeof(SelectState) <= kNoallocStateBytes, "state slot too small")
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
-// Device address of g_noalloc_scratch on the current device, looked up once per device.
+// Unique id of the context current on this thread (0 when none is current or the driver's
+// entry points are unavailable).  A device reset or a rebuilt primary context gets a new id
+// and a new load of this library's module, hence a new address of g_noalloc_scratch.  The
+// two driver calls are reached through the runtime's entry-point query, so the library does
+// not link the driver library itself.
+unsigned long long current_context_id() {
+  typedef CUresult (*GetCurrent)(CUcontext*);
+  typedef CUresult (*GetId)(CUcontext, unsigned long long*);
+  static GetCurrent get_current = nullptr;
+  static GetId get_id = nullptr;
+  static bool looked_up = false;
+  if (!looked_up) {
+    looked_up = true;
+    void* f1 = nullptr;
+    void* f2 = nullptr;
+    cudaDriverEntryPointQueryResult q1, q2;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f1, 12000, cudaEnableDefault, &q1) == cudaSuccess &&
+        cudaGetDriverEntryPointByVersion("cuCtxGetId", &f2, 12000, cudaEnableDefault, &q2) == cudaSuccess &&
+        q1 == cudaDriverEntryPointSuccess && q2 == cudaDriverEntryPointSuccess) {
+      get_current = reinterpret_cast<GetCurrent>(f1);
+      get_id = reinterpret_cast<GetId>(f2);
+    }
+    cudaGetLastError();
+  }
+  if (!get_current || !get_id) return 0;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Device address of g_noalloc_scratch on the current device.  It is looked up once per
+// device and context (cudaGetSymbolAddress, a host-side query that allocates nothing) and
+// cached under the context's id, so a reset device gets a fresh lookup.  Without a readable
+// id the lookup runs on every call.
 cudaError_t noalloc_scratch(void** out) {
+  struct Entry {
+    unsigned long long ctx;
+    void* addr;
+  };
   static std::mutex mu;
-  static void* addr[64] = {};
+  static Entry cache[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return e;
-    addr[dev] = p;
+  unsigned long long ctx = current_context_id();
+  if (ctx != 0 && cache[dev].ctx == ctx && cache[dev].addr) {
+    *out = cache[dev].addr;
+    return cudaSuccess;
   }
-  *out = addr[dev];
+  void* p = nullptr;
+  e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // also makes the device's context current
+  if (e != cudaSuccess) return e;
+  if (ctx == 0) ctx = current_context_id();
+  cache[dev].ctx = ctx;
+  cache[dev].addr = ctx ? p : nullptr;
+  *out = p;
   return cudaSuccess;
 }
 
@@ -1161,7 +1304,7 @@ cudaError_t launch_query_topk_noalloc(const float* merged, const HashCoeffs& h, 
   const int nb = (int)nseg;
   if (qp.vec) launch(k_count<true>, nb, kSegThreads, s, est_out, d, st, blk_gt, blk_eq);
   else launch(k_count<false>, nb, kSegThreads, s, est_out, d, st, blk_gt, blk_eq);
-  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, nseg, st, blk_base, blk_eqx, (uint32_t*)nullptr, d, (uint32_t)k);
+  launch(k_scan, 1, kScanThreads, s, blk_gt, blk_eq, nseg, st, blk_base, blk_eqx);
   if (qp.vec) launch(k_write<true>, nb, kSegThreads, s, est_out, d, st, blk_base, blk_eqx, idx_out, k);
   else launch(k_write<false>, nb, kSegThreads, s, est_out, d, st, blk_base, blk_eqx, idx_out, k);
   return cudaGetLastError();

@@ -256,14 +256,45 @@ def test_topk_large_plateau(gs, H, d, k, nonzero):
         run.close()
 
 
-@pytest.mark.parametrize("r,scale", [(5, 1e-3), (5, 0.97), (5, 30.0), (4, 1e-3), (7, 0.5), (3, 1e-3)])
-def test_pruned_query_matches_full_query(gs, H, r, scale):
-    """Queries whose estimate stays in the workspace skip rows below a prune key taken from the
-    sketch's previous query (same d and k).  After a query on x, the sketch is refilled with
-    scale * x (other noise), and queried again internally: with scale = 1e-3 or 0.5 the prune key
-    lies above the new threshold and the repair pass must restore every pruned estimate; with
-    0.97 or 30 pruning is safe.  Either way the selection equals the full query's exactly, every
-    selected estimate is exact, and every pruned (-0.0) one is below the k-th largest |est|."""
+SAMPLE_PERIOD = 256   # the query's prune-key sample: the first four coordinates of every 256
+
+
+def _prune_input(rng, d, k, adversarial):
+    """A vector with k heavy coordinates over N(0, 1e-2^2) noise.  Natural: the heavy
+    coordinates sit at random positions.  Adversarial: all of them sit on the query's sample
+    (coordinates i with i mod 256 < 4), with magnitudes spread over two decades, so that the
+    sample's rank puts the prune key far above the k-th largest |est| and the repair must run."""
+    x = (rng.standard_normal(d) * 1e-2).astype(np.float32)
+    if adversarial:
+        pos = (np.arange(k) // 4) * SAMPLE_PERIOD + (np.arange(k) % 4)
+        assert pos[-1] < d
+    else:
+        pos = rng.choice(d, k, replace=False)
+    mag = np.exp(rng.uniform(0.0, np.log(100.0), k)).astype(np.float32)
+    x[pos] = mag * rng.choice(np.array([-1.0, 1.0], np.float32), k)
+    return x
+
+
+def _check_pruned_against_full(H, got, e_int, want, e, k):
+    assert np.array_equal(got, want), "selections differ"
+    H.check_selection_exact(got, e, k)
+    pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
+    exact = e_int.view(np.uint32) == e.view(np.uint32)
+    assert np.all(pruned | exact)
+    tau = np.sort(np.abs(e))[-k]
+    assert np.all(np.abs(e[pruned]) < tau) and not pruned[got].any()
+    return pruned
+
+
+@pytest.mark.parametrize("r,adversarial", [(5, False), (5, True), (4, False), (4, True), (7, False), (7, True),
+                                           (3, False), (3, True)])
+def test_pruned_query_matches_full_query(gs, H, r, adversarial):
+    """Queries whose estimate stays in the workspace skip rows below a prune key that the query
+    takes from a strided sample of its own estimate.  On natural input the key is safe and most
+    coordinates stop after r/2 + 1 rows; on adversarial input (every heavy coordinate on the
+    sample) the key lies above the k-th largest |est|, and the repair pass must restore every
+    skipped estimate.  Either way the selection equals the full query's exactly, every selected
+    estimate is exact, and every skipped (-0.0) one lies below the k-th largest |est|."""
     d, c, k, seed = 4_200_007, 1 << 16, 4000, 40 + r      # pruning applies from d = 2^22
     rng = np.random.default_rng(seed)
     sk = gs.gs_sketch_create(r, c, seed, 1, 0)
@@ -273,32 +304,58 @@ def test_pruned_query_matches_full_query(gs, H, r, scale):
         idx = torch.empty(k, dtype=torch.int64, device="cuda")
         idx_full = torch.empty(k, dtype=torch.int64, device="cuda")
         est_full = torch.empty(d, dtype=torch.float32, device="cuda")
-        for t, sc in enumerate([1.0, scale, scale]):
-            x = (rng.standard_normal(d) * 1e-2).astype(np.float32)
-            x[rng.choice(d, 12_000, replace=False)] *= 40
-            x = (x * np.float32(sc)).astype(np.float32)
-            gs.gs_sketch_zero(sk)
-            gs.gs_sketch_insert(sk, 0, _dev(x), d)
-            gs.gs_sketch_merge_tree(sk, 1)
-            gs.gs_query_topk(sk, d, k, idx, None, ws)          # internal estimate: may prune
+        x = _prune_input(rng, d, k, adversarial)
+        gs.gs_sketch_zero(sk)
+        gs.gs_sketch_insert(sk, 0, _dev(x), d)
+        gs.gs_sketch_merge_tree(sk, 1)
+        for t in range(2):   # the same query twice: nothing carries over from the first
+            gs.gs_query_topk(sk, d, k, idx, None, ws)           # internal estimate: may prune
             torch.cuda.synchronize()
             got, e_int = H.host(idx).copy(), H.host(est_int).copy()
             gs.gs_query_topk(sk, d, k, idx_full, est_full, ws)  # caller's estimate: every row
             torch.cuda.synchronize()
-            want, e = H.host(idx_full), H.host(est_full)
-            assert np.array_equal(got, want), f"query {t}: selections differ"
-            H.check_selection_exact(got, e, k)
-            pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
-            exact = e_int.view(np.uint32) == e.view(np.uint32)
-            assert np.all(pruned | exact)
-            tau = np.sort(np.abs(e))[-k]
-            assert np.all(np.abs(e[pruned]) < tau) and not pruned[got].any()
-            if t == 0:
-                assert not pruned.any()                         # no record yet: nothing pruned
-            if t == 2:
-                assert pruned.mean() > 0.3                      # same scale as the query before
+            pruned = _check_pruned_against_full(H, got, e_int, H.host(idx_full), H.host(est_full), k)
+            if adversarial:
+                assert not pruned.any(), "the repair left skipped estimates"
+            else:
+                assert pruned.mean() > 0.5, f"only {pruned.mean():.3f} of the coordinates skipped rows"
     finally:
         gs.gs_sketch_destroy(sk)
+
+
+def test_pruned_queries_on_two_streams(gs, H):
+    """Queries of one sketch on two streams at once, each with its own workspace, one on natural
+    and one on adversarial data (a second sketch), interleaved launch after launch: a query keeps
+    its prune key in its own workspace, so every selection equals the full query's."""
+    d, r, c, k = 4_200_007, 5, 1 << 16, 4000
+    rng = np.random.default_rng(17)
+    sks = [gs.gs_sketch_create(r, c, 17, 1, 0) for _ in range(2)]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    try:
+        for sk, adv in zip(sks, (False, True)):
+            gs.gs_sketch_insert(sk, 0, _dev(_prune_input(rng, d, k, adv)), d)
+            gs.gs_sketch_merge_tree(sk, 1)
+        wss = [torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda") for _ in range(4)]
+        want = []
+        for sk in sks:
+            idx_full = torch.empty(k, dtype=torch.int64, device="cuda")
+            gs.gs_query_topk(sk, d, k, idx_full, torch.empty(d, dtype=torch.float32, device="cuda"), wss[0])
+            torch.cuda.synchronize()
+            want.append(H.host(idx_full).copy())
+        torch.cuda.synchronize()
+        idxs = [[torch.empty(k, dtype=torch.int64, device="cuda") for _ in range(12)] for _ in range(2)]
+        for n in range(12):
+            for q in range(2):
+                # stream q alternates between the two sketches; each stream uses its own workspaces
+                gs.gs_query_topk(sks[(n + q) % 2], d, k, idxs[q][n], None, wss[2 * q + (n % 2)], None,
+                                 streams[q])
+        torch.cuda.synchronize()
+        for q in range(2):
+            for n in range(12):
+                assert np.array_equal(H.host(idxs[q][n]), want[(n + q) % 2]), f"stream {q}, query {n}"
+    finally:
+        for sk in sks:
+            gs.gs_sketch_destroy(sk)
 
 
 def test_no_pruning_below_4m_coordinates(gs, H):
