@@ -2,8 +2,9 @@
 
 One step = the whole hot path for P simulated workers on one GPU: accumulate + Count
 Sketch insert (fused), tree merge, median query + top-k, gather-and-zero.  The metric is
-gradient coordinates per second, P * d * steps / time, for the ResNet-18-sized workload
-(d = 11,173,962, P = 8, r = 5, c = 2^17, k = 11,200) unless --config names another.
+gradient coordinates per second, P * d * steps / time.  The headline workload is the
+ResNet-50-sized one (d = 25,557,032, P = 8, r = 5, c = 2^18, k = 25,600) unless --config
+names another; `per_config` in the same JSON line times every workload of the suite.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
 
@@ -19,7 +20,6 @@ import argparse
 import hashlib
 import json
 import os
-import re
 import statistics
 import subprocess
 import sys
@@ -35,12 +35,16 @@ import workloads  # noqa: E402
 
 METRIC = "gradient coords/s through accumulate+sketch+merge+top-k at P=8; % HBM roofline"
 UNIT = "coords/s"
-K1_SOURCE = os.path.join(ROOT, "paper_2108_06004_gb300", "csrc", "k_insert.cu")
-PROFILE_DIR = os.path.join(ROOT, "profiles")
+DEFAULT_CONFIG = "resnet50"
+CSRC = os.path.join(ROOT, "paper_2108_06004_gb300", "csrc")
+TRAFFIC_JSON = os.path.join(ROOT, "profiles", "traffic.json")
 CPU_SAMPLE_D = 1 << 22   # coordinates per worker in one bounded oracle step (CPU baseline)
 REF_BUDGET_S = 120.0     # oracle seconds for a whole --impl reference run
 ORACLE_S_PER_COORD = 1.7e-7  # oracle seconds per worker-coordinate (sizes the reference samples)
-
+L2_BYTES = 126 << 20     # GB300 L2; inputs below twice this are flushed between timed steps
+PER_CONFIG_STEPS = {"tiny-2^20": 300, "resnet18": 300, "resnet50": 100, "vgg16": 5, "bert-large": 3}
+PRUNE_MIN_DIM = 1 << 22  # the library skips query rows from this dimension on
+SAMPLE_PERIOD = 256      # ... with a prune-key sample of the first four of every 256 coordinates
 
 VARIANTS = {
     "error_feedback": "S1-S6: per-worker momentum and error vectors, exact second round",
@@ -52,12 +56,12 @@ HEAVYMIX_FILL_SEED = 0x5EED5EED
 LR = 0.01
 
 
-def parse_args():
+def parse_args(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--config", default="resnet18", choices=sorted(workloads.CONFIGS))
+    ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(workloads.CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--variant", default="error_feedback", choices=list(VARIANTS),
                     help="which form of the step to time (the default is the headline path)")
@@ -65,9 +69,26 @@ def parse_args():
                     help="one library call per kernel instead of a captured plan per step")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-config", action="store_true", help="time only the headline workload")
     ap.add_argument("--profile-steps", action="store_true",
-                    help="short run for a profiler: no e2e, no CPU baseline, no clocks")
-    return ap.parse_args()
+                    help="short run for a profiler: no e2e, no CPU baseline, no clocks, no probes, no per-config")
+    ap.add_argument("--d", type=int, default=0,
+                    help="profiling a small case: the workload's first D coordinates (its leading blocks, the "
+                         "last one cut), same P, r, c and k scaled with D; implies --profile-steps")
+    return ap.parse_args(argv)
+
+
+def shrink(w, d: int):
+    """The workload restricted to its first d coordinates (blocks cut at d; k scaled with d)."""
+    import dataclasses
+    blocks, tot = [], 0
+    for b in w.blocks:
+        if tot >= d:
+            break
+        blocks.append(min(b, d - tot))
+        tot += blocks[-1]
+    return dataclasses.replace(w, d=d, k=max(1, round(w.k * d / w.d)), block_sizes=tuple(blocks),
+                               name=f"{w.name}@d={d}")
 
 
 def measured_peaks():
@@ -142,22 +163,24 @@ class ClockSampler:
                 "window_s": round(self.t1 - self.t0, 3)}
 
 
-# ---- profile summary (ncu traffic) -------------------------------------------------------
+# ---- ncu traffic ------------------------------------------------------------------------
 
-def k1_traffic_per_launch(workload: str):
-    """DRAM bytes per launch of the fused accumulate+insert kernel on this workload from the
-    committed ncu summary (profiles/accumulate_insert_<workload>.md), if there is one and it
-    was taken on the current kernel source (else None)."""
+def source_sha16(name: str) -> str:
+    return hashlib.sha256(open(os.path.join(CSRC, name), "rb").read()).hexdigest()[:16]
+
+
+def measured_traffic(kernel: str, workload: str):
+    """DRAM bytes (read + write) per launch of `kernel` on `workload` from profiles/traffic.json
+    (written from one ncu capture, scaled to a full launch where the capture was smaller), if
+    it was taken on the current source of the kernel's file; else None."""
     try:
-        text = open(os.path.join(PROFILE_DIR, f"accumulate_insert_{workload}.md")).read()
-    except OSError:
+        with open(TRAFFIC_JSON) as f:
+            entry = json.load(f)["kernels"][kernel][workload]
+    except (OSError, KeyError, ValueError):
         return None
-    src = hashlib.sha256(open(K1_SOURCE, "rb").read()).hexdigest()[:16]
-    m_sha = re.search(r"kernel source sha256\[:16\]:\s*`?([0-9a-f]{16})", text)
-    m_tr = re.search(r"traffic per full launch \(bytes\):\s*`?([0-9.eE+]+)", text)
-    if not m_sha or not m_tr or m_sha.group(1) != src:
+    if entry.get("source_sha16") != source_sha16(entry["source"]):
         return None
-    return float(m_tr.group(1))
+    return entry.get("dram_bytes_per_full_launch")
 
 
 # ---- ranks --------------------------------------------------------------------------------
@@ -183,12 +206,450 @@ def whole_job_rate(world: int, P: int, d: int, steps: int, max_seconds: float) -
     return world * P * d * steps / max_seconds
 
 
-# ---- our arm -----------------------------------------------------------------------------
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
 
 def gpu_uuid(dev) -> str:
     import torch
     u = str(torch.cuda.get_device_properties(dev).uuid)
     return u if u.startswith("GPU-") else "GPU-" + u
+
+
+# ---- one workload ---------------------------------------------------------------------------
+
+def _event_pair(record):
+    import torch
+    if not record:
+        return None
+    return torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+
+class Runner:
+    """Everything one workload's timed steps need: state, sketches, workspace, gradients and,
+    unless eager, one plan (CUDA graph) per gradient buffer set.
+
+    Workloads whose P workers are all resident draw a pool of fresh gradient sets (one per step
+    of the workload, as many as fit 24 GB), cycled over the timed steps.  A workload with a
+    worker batch (BERT-large: 32 workers, 8 resident) streams: every step, for each batch, the
+    batch's fresh gradients are drawn on the device into one shared buffer set (timed with
+    their own events, outside the insert's) and then inserted; such steps run eagerly."""
+
+    def __init__(self, gs, w, variant, eager, rank, dev, stream, steps_needed, want_host_pool):
+        import torch
+        self.gs, self.w, self.variant, self.dev, self.stream = gs, w, variant, dev, stream
+        self.rank = rank
+        P, d, r, c, k = w.P, w.d, w.r, w.c, w.k
+        self.streamed = bool(w.worker_batch) and w.worker_batch < P
+        self.batch = w.worker_batch if self.streamed else P
+        self.host_pool, self.dev_pool = [], []
+        if self.streamed:
+            self.gbuf = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(self.batch)]
+            self.nsteps_pool = 1
+        else:
+            step_bytes = P * d * 4
+            self.nsteps_pool = max(1, min(w.steps, steps_needed, (24 << 30) // step_bytes))
+            host_gen = step_bytes <= (1 << 30)
+            for t in range(self.nsteps_pool):
+                if host_gen:
+                    gl = workloads.make_gradients(w, t, replica_workers(rank, P))
+                    hp = [torch.from_numpy(g).pin_memory() for g in gl]
+                    if want_host_pool:
+                        self.host_pool.append(hp)
+                    self.dev_pool.append([g.to(dev, non_blocking=True) for g in hp])
+                else:
+                    self.dev_pool.append([workloads.make_gradient_torch(w, t, q, torch.empty(d, device=dev))
+                                          for q in replica_workers(rank, P)])
+            if want_host_pool and not host_gen:
+                self.host_pool = [[g.cpu().pin_memory() for g in self.dev_pool[0]]]
+        self.us = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
+        self.es = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
+        gs = self.gs
+        self.sk = gs.gs_sketch_create(r, c, 20210813, P, 0)
+        info = gs.gs_sketch_info(self.sk)
+        self.W, self.rpp = info["group_width"], info["rows_per_pass"]
+        self.groups = (P + self.W - 1) // self.W
+        self.passes = -(-r // self.rpp)
+        ws_bytes = gs.gs_step_workspace_size(d, k)
+        if variant == "heavymix":
+            ws_bytes = max(ws_bytes, gs.gs_query_heavymix_workspace_size(d, k))
+        self.ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+        self.qws_bytes = gs.gs_query_topk_workspace_size(d, k)
+        self.l2sq = torch.empty(1, dtype=torch.float64, device=dev)
+        self.weights = torch.zeros(d, dtype=torch.float32, device=dev) if variant in ("train", "sketched_state") \
+            else None
+        self.sk_u = self.sk_e = None
+        if variant == "sketched_state":
+            self.sk_u = gs.gs_sketch_create(r, c, 20210813, 1, 0)
+            self.sk_e = gs.gs_sketch_create(r, c, 20210813, 1, 0)
+            gs.gs_sketch_zero(self.sk_u)
+            gs.gs_sketch_zero(self.sk_e)
+        self.idx = torch.empty(k, dtype=torch.int64, device=dev)
+        self.vals = torch.empty(k, dtype=torch.float32, device=dev)
+        self.use_plan = (not eager or variant == "sketched_state") and not self.streamed
+        self.plans = []
+        flags = gs.GS_PLAN_TIME_INSERT | gs.GS_PLAN_TIME_QUERY
+        if self.use_plan:
+            for grads in self.dev_pool:
+                if variant == "sketched_state":
+                    self.plans.append(gs.gs_sketched_state_plan_create(
+                        self.sk, self.sk_u, self.sk_e, grads, d, w.rho, k, self.idx, self.vals, self.weights, LR,
+                        self.ws, flags=flags))
+                elif variant == "heavymix":
+                    self.plans.append(gs.gs_heavymix_step_plan_create(
+                        self.sk, self.us, self.es, grads, d, w.rho, k, HEAVYMIX_FILL_SEED, self.idx, self.vals,
+                        self.l2sq, self.ws, flags=flags))
+                else:
+                    self.plans.append(gs.gs_step_plan_create(self.sk, self.us, self.es, grads, d, w.rho, k, self.idx,
+                                                             self.vals, None, self.weights, LR, self.ws, flags=flags))
+        self.ev = {"insert": [], "query": [], "gen": []}   # eager: per step, a list of (begin, end) pairs
+
+    def step(self, t, record):
+        gs, w, s = self.gs, self.w, self.stream
+        d, k, rho = w.d, w.k, w.rho
+        if self.use_plan:
+            gs.gs_plan_launch(self.plans[t % self.nsteps_pool], s)
+            return
+        if self.variant == "sketched_state":
+            raise RuntimeError("the sketched state always runs as a plan")
+        gs.gs_sketch_zero(self.sk, s)
+        if self.streamed:
+            ins_pairs, gen_pairs = [], []
+            for b0 in range(0, w.P, self.batch):
+                gen = _event_pair(record)
+                if gen:
+                    gen[0].record(s)
+                for q in range(self.batch):
+                    workloads.make_gradient_torch(w, t, self.rank * w.P + b0 + q, self.gbuf[q])
+                if gen:
+                    gen[1].record(s)
+                    gen_pairs.append(gen)
+                ins = _event_pair(record)
+                if ins:
+                    ins[0].record(s)
+                gs.gs_accumulate_insert(self.sk, b0, self.us[b0:b0 + self.batch], self.es[b0:b0 + self.batch],
+                                        self.gbuf, d, rho, s)
+                if ins:
+                    ins[1].record(s)
+                    ins_pairs.append(ins)
+            if record:
+                self.ev["insert"].append(ins_pairs)
+                self.ev["gen"].append(gen_pairs)
+        else:
+            ins = _event_pair(record)
+            if ins:
+                ins[0].record(s)
+            gs.gs_accumulate_insert(self.sk, 0, self.us, self.es, self.dev_pool[t % self.nsteps_pool], d, rho, s)
+            if ins:
+                ins[1].record(s)
+                self.ev["insert"].append([ins])
+        gs.gs_sketch_merge_tree(self.sk, w.P, s)
+        q = _event_pair(record)
+        if q:
+            q[0].record(s)
+        if self.variant == "heavymix":
+            gs.gs_query_heavymix(self.sk, d, k, HEAVYMIX_FILL_SEED, self.idx, None, self.l2sq, self.ws, None, s)
+        else:
+            gs.gs_query_topk(self.sk, d, k, self.idx, None, self.ws, self.qws_bytes, s)
+        if q:
+            q[1].record(s)
+            self.ev["query"].append([q])
+        if self.variant == "train":
+            gs.gs_gather_zero_update(self.us, self.es, d, self.idx, k, self.vals, self.weights, LR, s)
+        else:
+            gs.gs_gather_and_zero(self.us, self.es, d, self.idx, k, self.vals, s)
+
+    def phase_times(self, n_timed_by_plan):
+        """Mean ms of the insert phase, the median query (plans) and the selection (plans), or
+        of the whole query + selection (eager), and of gradient generation (streamed)."""
+        def mean(x):
+            return sum(x) / len(x) if x else None
+        if self.use_plan:
+            ins, qry, sel = [], [], []
+            for i, plan in enumerate(self.plans):
+                n = n_timed_by_plan[i]
+                if n:
+                    ins += self.gs.gs_plan_insert_times(plan, n)
+                    a, b = self.gs.gs_plan_query_times(plan, n)
+                    qry += a
+                    sel += b
+            return {"insert": mean(ins), "query": mean(qry), "select": mean(sel), "query_select": None, "gen": None,
+                    "n": len(ins)}
+        def per_step(phase):   # each step's pairs summed (a streamed step has one per batch)
+            return [sum(a.elapsed_time(b) for a, b in pairs) for pairs in self.ev[phase]]
+        ins = per_step("insert")
+        return {"insert": mean(ins), "query": None, "select": None, "query_select": mean(per_step("query")),
+                "gen": mean(per_step("gen")), "n": len(ins)}
+
+    def pruned_fraction(self):
+        """Fraction of coordinates whose last query stopped after r/2 + 1 rows (stored -0.0)."""
+        import torch
+        d = self.w.d
+        est = self.ws[: 4 * d].view(torch.int32)
+        return float((est == -2**31).sum().item()) / d
+
+    def close(self):
+        for plan in self.plans:
+            self.gs.gs_plan_destroy(plan)
+        self.plans = []
+        for sk in (self.sk, self.sk_u, self.sk_e):
+            if sk:
+                self.gs.gs_sketch_destroy(sk)
+        self.sk = self.sk_u = self.sk_e = None
+
+
+def launches_per_step(run: Runner, variant: str) -> int:
+    """Kernels of the library launched per step: insert (one per group and row pass, and per
+    worker batch), merge, the query and selection, the gather (sketched state: its own)."""
+    w = run.w
+    prunes = variant != "heavymix" and w.d >= PRUNE_MIN_DIM and w.r >= 3 and (w.c & (w.c - 1)) == 0
+    inserts = run.groups * run.passes
+    if variant == "heavymix":
+        query = 4 + 6                                 # sumsq, theta, query, keys + selection
+    else:
+        query = 1 + 6 + (2 if prunes else 0)          # query + selection (+ sample and repair check)
+    tail = 6 if variant == "sketched_state" else 1
+    return inserts + 1 + query + tail
+
+
+def time_steps(run: Runner, steps: int, warmup: int, world: int, dev, sampler=None, flush=None):
+    """Run warm-up steps (every plan at least once), then time `steps` steps.  Without `flush`
+    the timed region is bracketed by events on the stream; with it (inputs that fit in L2), a
+    buffer larger than L2 is written before every timed step, outside that step's events."""
+    import torch
+    s = run.stream
+    n_warm = max(warmup, len(run.plans))
+    for t in range(n_warm):
+        run.step(t, False)
+    torch.cuda.synchronize()
+    for k in run.ev:
+        run.ev[k].clear()
+    barrier(world)
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark_begin()
+    if flush is None:
+        start = torch.cuda.Event(enable_timing=True)
+        end = torch.cuda.Event(enable_timing=True)
+        start.record(s)
+        for t in range(steps):
+            run.step(warmup + t, True)
+        end.record(s)
+        torch.cuda.synchronize()
+        elapsed = start.elapsed_time(end)
+    else:
+        pairs = []
+        for t in range(steps):
+            flush.add_(1)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            run.step(warmup + t, True)
+            b.record(s)
+            pairs.append((a, b))
+        torch.cuda.synchronize()
+        elapsed = sum(a.elapsed_time(b) for a, b in pairs)
+    barrier(world)
+    if sampler:
+        sampler.mark_end()
+    elapsed = dist_max(elapsed, dev)
+    n_by_plan = [sum(1 for t in range(steps) if (warmup + t) % run.nsteps_pool == i) for i in range(len(run.plans))]
+    return elapsed, n_warm, n_by_plan
+
+
+def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dict, pruned: float):
+    """The insert-phase roofline (HBM, with the measured request ceiling as co-bound) and the
+    median query's (L1->L2 requests against the measured gather ceiling; HBM bytes alongside)."""
+    w = run.w
+    P, d, r = w.P, w.d, w.r
+    per_wc = 4.0 if variant == "sketched_state" else 20.0
+    moved_wc = per_wc + 4.0 * (run.passes - 1)
+    phase_s = ph["insert"] / 1e3
+    phase_bytes = per_wc * P * d
+    k1_gbs = phase_bytes / phase_s / 1e9
+    cells = d * r * run.groups
+    nl = run.groups * run.passes * (w.P // run.batch if run.streamed else 1)
+    k1 = {
+        "kernel": ("k_accumulate_insert_coop (insert only" if variant == "sketched_state" else
+                   "k_accumulate_insert_coop (fused S1+S2") + f", W={run.W}), the insert phase of a step: "
+                  f"{run.groups} group(s) x {run.passes} row pass(es)",
+        "row_passes": run.passes, "groups": run.groups, "launches_per_phase": nl,
+        "algorithmic_bytes_per_worker_coord": per_wc, "moved_bytes_per_worker_coord": moved_wc,
+        "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+        "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
+        "frac_of_nominal_8000_GBps": round(k1_gbs / 8000.0, 4),
+        "traffic": (measured_traffic("k_accumulate_insert_coop", w.name)
+                    if variant == "error_feedback" and nl == 1 else None),
+        "algorithmic_bytes_per_launch": phase_bytes / nl if nl == 1 else None,
+        "algorithmic_bytes_per_phase": phase_bytes,
+        "avg_launch_ms": round(ph["insert"] / nl, 4),
+        "avg_phase_ms": round(ph["insert"], 4),
+        "timed_phases": ph["n"],
+        "timing": "event-record nodes inside the step's CUDA graph" if run.use_plan else "CUDA events around the call",
+    }
+    ceil_ms = probes.get("insert_ms")
+    k1["co_bound"] = {
+        "kind": "SM->L2 requests: one cell reduction per (coordinate, row, group) plus the u, e stores and the loads",
+        "probe": "gs_insert_request_ceiling: the same kernels, grids, buckets and reductions with every vector access "
+                 "folded into an L2-resident window (no HBM traffic)",
+        "cell_updates_per_phase": cells,
+        "achieved_G_cells_per_s": round(cells / phase_s / 1e9, 1),
+        "peak_ms": None if ceil_ms is None else round(ceil_ms, 4),
+        "peak": None if ceil_ms is None else round(phase_bytes / (ceil_ms / 1e3) / 1e9, 1),
+        "unit": "GB/s of algorithmic bytes",
+        "frac": None if ceil_ms is None else round(ceil_ms / ph["insert"], 4),
+        "peak_frac_of_hbm": None if ceil_ms is None else round(phase_bytes / (ceil_ms / 1e3) / 1e9 / peaks["hbm_gbs"], 4),
+    }
+    q = None
+    q_ms = ph["query"]
+    if q_ms is not None and variant != "heavymix":
+        kf = r // 2 + 1
+        prunes = d >= PRUNE_MIN_DIM and r >= 3 and (w.c & (w.c - 1)) == 0
+        nq = (d + 3) // 4
+        n_s = 4 * ((nq + SAMPLE_PERIOD // 4 - 1) // (SAMPLE_PERIOD // 4)) if prunes else 0
+        requests = d * kf + d * (r - kf) * (1.0 - pruned) + n_s * r
+        g_ms = probes.get("query_ms")
+        ach = requests / (q_ms / 1e3) / 1e9
+        q = {
+            "kernel": f"k_qsample + k_query<{r}> + k_repair (median query, S4)" if prunes else f"k_query<{r}> (S4)",
+            "bound": "L1->L2 requests (scattered 4-byte reads of the merged table)",
+            "avg_ms": round(q_ms, 4), "pruned_fraction": round(pruned, 4),
+            "requests_per_step": requests, "requests_per_coord": round(requests / d, 3),
+            "achieved_G_requests_per_s": round(ach, 1),
+            "peak_G_requests_per_s": None if g_ms is None else round(d * r / (g_ms / 1e3) / 1e9, 1),
+            "peak_probe": "gs_query_request_ceiling: the query's loads of all r rows, no median or store",
+            "frac": None if g_ms is None else round(ach / (d * r / (g_ms / 1e3) / 1e9), 4),
+            "time_vs_full_read_ceiling": None if g_ms is None else round(g_ms / q_ms, 4),
+            "hbm": {"algorithmic_bytes": 4 * d, "achieved_GBps": round(4 * d / (q_ms / 1e3) / 1e9, 1),
+                    "frac": round(4 * d / (q_ms / 1e3) / 1e9 / peaks["hbm_gbs"], 4)},
+            "select_ms": None if ph["select"] is None else round(ph["select"], 4),
+        }
+    return k1, q
+
+
+def probe_ceilings(run: Runner, reps: int = 3) -> dict:
+    """The insert's and the query's measured request ceilings (medians of `reps`), run outside
+    the timed region; the insert probe leaves the worker tables unspecified, and every step
+    zeroes them first."""
+    gs = run.gs
+    out = {}
+    if run.W >= 4 and (run.w.c & (run.w.c - 1)) == 0:
+        import torch
+        win = torch.empty(max(gs.gs_insert_request_ceiling_window_size(run.sk), 1 << 16), dtype=torch.uint8,
+                          device=run.dev)
+        out["insert_ms"] = statistics.median(gs.gs_insert_request_ceiling(run.sk, run.w.d, win, None, run.stream)
+                                             for _ in range(reps))
+        out["query_ms"] = statistics.median(gs.gs_query_request_ceiling(run.sk, run.w.d, win, None, run.stream)
+                                            for _ in range(reps))
+        del win
+    return out
+
+
+def measure(gs, w, variant, eager, steps, warmup, world, rank, dev, stream, peaks, peak_kind, sampler=None,
+            want_e2e=False, probes=True):
+    """Time one workload; returns (summary dict, Runner still open for e2e)."""
+    import torch
+    want_host = want_e2e and variant == "error_feedback"
+    run = Runner(gs, w, variant, eager, rank, dev, stream, steps + warmup, want_host)
+    flush = None
+    streamed_bytes = w.P * w.d * 12
+    if streamed_bytes < 2 * L2_BYTES:
+        flush = torch.zeros(64 << 20, dtype=torch.float32, device=dev)   # 256 MB, twice the L2
+    torch.cuda.synchronize()
+    elapsed_ms, n_warm, n_by_plan = time_steps(run, steps, warmup, world, dev, sampler, flush)
+    ph = run.phase_times(n_by_plan)
+    pruned = run.pruned_fraction() if variant != "heavymix" else 0.0
+    pr = probe_ceilings(run) if probes else {}
+    k1, q = rooflines(run, variant, ph, peaks, peak_kind, pr, pruned)
+    value = whole_job_rate(world, w.P, w.d, steps, elapsed_ms / 1e3)
+    res = {
+        "value": value, "ms_per_step": round(elapsed_ms / steps, 4), "steps": steps, "warmup_steps_run": n_warm,
+        "launch": "plan" if run.use_plan else "eager",
+        "l2": ("flushed before every timed step (256 MB write, outside the step's events)" if flush is not None else
+               f"inputs larger than L2 ({streamed_bytes / 1e9:.2f} GB of g,u,e streamed per step)"),
+        "gpu_launches_per_step": launches_per_step(run, variant),
+        "roofline": k1, "roofline_query": q,
+        "insert_share_of_step": round(ph["insert"] / (elapsed_ms / steps), 3),
+    }
+    if run.streamed:
+        res["streaming"] = {
+            "worker_batch": run.batch,
+            "gradient_generation_ms_per_step": None if ph["gen"] is None else round(ph["gen"], 3),
+            "note": "every step draws fresh gradients for each batch of resident workers into one shared device "
+                    "buffer set, then inserts the batch; generation is inside the step, outside the insert's events",
+        }
+        if ph["gen"] is not None:
+            res["ms_per_step_without_generation"] = round(elapsed_ms / steps - ph["gen"], 4)
+    if ph["query_select"] is not None:
+        res["query_and_selection_ms"] = round(ph["query_select"], 4)
+    del flush
+    return res, run
+
+
+def e2e_measure(gs, run: Runner, steps, warmup, world, dev):
+    """End to end through the public API with host buffers: a host plan per gradient set (the
+    uploads where needed, the step and the download of idx and vals are one graph), then a
+    stream synchronisation so that the host can read the step's result."""
+    import torch
+    w = run.w
+    P, d, k = w.P, w.d, w.k
+    s = run.stream
+    grad_dev = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(P)]
+    idx_h = torch.empty(k, dtype=torch.int64).pin_memory()
+    vals_h = torch.empty(k, dtype=torch.float32).pin_memory()
+    hplans = []
+    if run.use_plan:
+        hplans = [gs.gs_step_host_plan_create(run.sk, run.us, run.es, hb, grad_dev, d, w.rho, k, idx_h, vals_h, run.ws)
+                  for hb in run.host_pool]
+
+    def host_step(t):
+        if run.use_plan:
+            gs.gs_plan_launch(hplans[t % len(hplans)], s)
+            s.synchronize()
+        else:
+            gs.gs_step_host(run.sk, run.us, run.es, run.host_pool[t % len(run.host_pool)], grad_dev, d, w.rho, k,
+                            idx_h, vals_h, run.ws, None, s)
+
+    for t in range(max(warmup, len(hplans))):   # every plan once, at least W steps
+        host_step(t)
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for t in range(steps):
+        host_step(warmup + t)
+    torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - t0
+    barrier(world)
+    e2e_s = dist_max(e2e_s, dev)
+    for hp in hplans:
+        gs.gs_plan_destroy(hp)
+    return {"value": whole_job_rate(world, P, d, steps, e2e_s), "unit": UNIT, "h2d_bytes_per_step": P * d * 4,
+            "d2h_bytes_per_step": k * (8 + 4), "ms_per_step": round(e2e_s * 1e3 / steps, 4),
+            "call": "gs_step_host_plan_create + gs_plan_launch" if run.use_plan else "gs_step_host"}
+
+
+def short_summary(res: dict, w) -> dict:
+    k1, q = res["roofline"], res["roofline_query"]
+    out = {
+        "d": w.d, "P": w.P, "r": w.r, "c": w.c, "k": w.k, "steps": res["steps"], "launch": res["launch"],
+        "value": res["value"], "unit": UNIT, "ms_per_step": res["ms_per_step"], "l2": res["l2"],
+        "insert": {"avg_phase_ms": k1["avg_phase_ms"], "achieved": k1["achieved"], "frac": k1["frac"],
+                   "row_passes": k1["row_passes"], "groups": k1["groups"],
+                   "moved_bytes_per_worker_coord": k1["moved_bytes_per_worker_coord"],
+                   "request_ceiling_ms": k1["co_bound"]["peak_ms"], "frac_of_request_ceiling": k1["co_bound"]["frac"],
+                   "request_ceiling_frac_of_hbm": k1["co_bound"]["peak_frac_of_hbm"]},
+        "query": None if q is None else {"avg_ms": q["avg_ms"], "pruned_fraction": q["pruned_fraction"],
+                                          "achieved_G_requests_per_s": q["achieved_G_requests_per_s"],
+                                          "peak_G_requests_per_s": q["peak_G_requests_per_s"], "frac": q["frac"],
+                                          "select_ms": q["select_ms"]},
+        "gpu_launches_per_step": res["gpu_launches_per_step"],
+    }
+    for key in ("streaming", "ms_per_step_without_generation", "query_and_selection_ms"):
+        if key in res:
+            out[key] = res[key]
+    return out
 
 
 def run_ours(args):
@@ -210,252 +671,70 @@ def run_ours(args):
         if rank == 0 or world == 1:
             from paper_2108_06004_gb300 import _build
             _build.build()
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
+        barrier(world)
     gs.load_library()
-
-    w = workloads.get_config(args.config)
-    P, d, r, c, k, rho = w.P, w.d, w.r, w.c, w.k, w.rho
-    # Fresh gradients for each of the workload's steps (cycled if more steps are timed),
-    # as many steps as fit a 24 GB pool.  Replicas on different ranks draw different
-    # workers' gradients.  Large workloads are drawn on the device.
-    step_bytes = P * d * 4
-    nsteps_pool = max(1, min(w.steps, args.steps + args.warmup, (24 << 30) // step_bytes))
-    host_gen = step_bytes <= (1 << 30)
-    host_pool, dev_pool = [], []
-    for t in range(nsteps_pool):
-        if host_gen:
-            gl = workloads.make_gradients(w, t, replica_workers(rank, P))
-            host_pool.append([torch.from_numpy(g).pin_memory() for g in gl])
-            dev_pool.append([g.to(dev, non_blocking=True) for g in host_pool[-1]])
-        else:
-            dev_pool.append([workloads.make_gradient_torch(w, t, q, torch.empty(d, device=dev))
-                             for q in replica_workers(rank, P)])
-    if not host_gen and not args.no_e2e and not args.profile_steps:
-        host_pool = [[g.cpu().pin_memory() for g in dev_pool[0]]]
-    us = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
-    es = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
-    sk = gs.gs_sketch_create(r, c, 20210813, P, 0)
-    W = gs.gs_sketch_info(sk)["group_width"]
-    groups = (P + W - 1) // W
-    variant = args.variant
-    ws_bytes = gs.gs_step_workspace_size(d, k)
-    if variant == "heavymix":
-        ws_bytes = max(ws_bytes, gs.gs_query_heavymix_workspace_size(d, k))
-    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
-    qws_bytes = gs.gs_query_topk_workspace_size(d, k)
-    l2sq = torch.empty(1, dtype=torch.float64, device=dev)
-    weights = torch.zeros(d, dtype=torch.float32, device=dev) if variant in ("train", "sketched_state") else None
-    sk_u = sk_e = None
-    if variant == "sketched_state":
-        sk_u = gs.gs_sketch_create(r, c, 20210813, 1, 0)
-        sk_e = gs.gs_sketch_create(r, c, 20210813, 1, 0)
-        gs.gs_sketch_zero(sk_u)
-        gs.gs_sketch_zero(sk_e)
-    idx = torch.empty(k, dtype=torch.int64, device=dev)
-    vals = torch.empty(k, dtype=torch.float32, device=dev)
-    stream = torch.cuda.current_stream()
-    torch.cuda.synchronize()
-
-    # Plans (one CUDA graph per gradient buffer set, the insert phase timed by event nodes
-    # inside the graph) unless --eager asks for one library call per kernel.  HEAVYMIX has
-    # no plan form and always runs eagerly; the sketched state always runs as a plan.
-    use_plan = (not args.eager or variant == "sketched_state") and variant != "heavymix"
-    plans = []
-    if use_plan:
-        for grads in dev_pool:
-            if variant == "sketched_state":
-                plans.append(gs.gs_sketched_state_plan_create(sk, sk_u, sk_e, grads, d, rho, k, idx, vals, weights,
-                                                              LR, ws, flags=gs.GS_PLAN_TIME_INSERT))
-            else:
-                plans.append(gs.gs_step_plan_create(sk, us, es, grads, d, rho, k, idx, vals, None, weights, LR, ws,
-                                                    flags=gs.GS_PLAN_TIME_INSERT))
-    k1_events = []
-
-    def step(t, record):
-        if use_plan:
-            gs.gs_plan_launch(plans[t % nsteps_pool], stream)
-            return
-        grads = dev_pool[t % nsteps_pool]
-        if variant == "sketched_state":
-            gs.gs_sketched_state_step(sk, sk_u, sk_e, grads, d, rho, k, idx, vals, weights, LR, ws, None, stream)
-            return
-        gs.gs_sketch_zero(sk, stream)
-        if record:
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-        gs.gs_accumulate_insert(sk, 0, us, es, grads, d, rho, stream)
-        if record:
-            e1.record(stream)
-            k1_events.append((e0, e1))
-        gs.gs_sketch_merge_tree(sk, P, stream)
-        if variant == "heavymix":
-            gs.gs_query_heavymix(sk, d, k, HEAVYMIX_FILL_SEED, idx, None, l2sq, ws, None, stream)
-        else:
-            gs.gs_query_topk(sk, d, k, idx, None, ws, qws_bytes, stream)
-        if variant == "train":
-            gs.gs_gather_zero_update(us, es, d, idx, k, vals, weights, LR, stream)
-        else:
-            gs.gs_gather_and_zero(us, es, d, idx, k, vals, stream)
-
-    n_warm = max(args.warmup, len(plans))  # at least W steps, and every plan launched once
-    for t in range(n_warm):
-        step(t, False)
-    torch.cuda.synchronize()
-
-    clocks = None
-    sampler = None
-    if not args.profile_steps:
-        sampler = ClockSampler(gpu_uuid(dev))
-        sampler.start()
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
-    torch.cuda.synchronize()
-    if sampler:
-        sampler.mark_begin()
-    start = torch.cuda.Event(enable_timing=True)
-    end = torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for t in range(args.steps):
-        step(args.warmup + t, True)
-    end.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
-    if sampler:
-        sampler.mark_end()
-    elapsed_ms = dist_max(start.elapsed_time(end), dev)
-    if sampler:
-        clocks = sampler.stop()
-
-    # insert-phase durations of the timed steps: each covers all groups and row passes
-    if use_plan:
-        k1_ms = []
-        for i, plan in enumerate(plans):
-            n_timed = sum(1 for t in range(args.steps) if (args.warmup + t) % nsteps_pool == i)
-            if n_timed:
-                k1_ms += gs.gs_plan_insert_times(plan, n_timed)
-    else:
-        k1_ms = [a.elapsed_time(b) for a, b in k1_events]
-    value = whole_job_rate(world, P, d, args.steps, elapsed_ms / 1e3)
-
-    # Roofline of the dominant phase, the insert: 20 algorithmic HBM bytes per worker-
-    # coordinate for the fused accumulate + insert (read g, u, e; write u, e); for the
-    # sketched state, 4 (read g).  Tables larger than the L2 pass budget take several row
-    # passes, each after the first re-reading e (or g): those bytes are reported as moved,
-    # not counted as algorithmic.  One launch covers one group of W workers and one row pass,
-    # so a phase is `groups` x `passes` launches.
     peaks, peak_kind = measured_peaks()
-    rpp = gs.gs_sketch_info(sk)["rows_per_pass"]
-    passes = -(-r // rpp)
-    per_wc = 4.0 if variant == "sketched_state" else 20.0
-    moved_wc = per_wc + 4.0 * (passes - 1)
-    phase_s = (sum(k1_ms) / len(k1_ms)) / 1e3
-    phase_bytes = per_wc * P * d
-    k1_gbs = phase_bytes / phase_s / 1e9
-    cells = d * r * groups
-    roofline = {
-        "kernel": ("k_accumulate_insert_coop (insert only" if variant == "sketched_state" else
-                   "k_accumulate_insert_coop (fused S1+S2") + f", W={W}), the insert phase of a step: "
-                  f"{groups} group(s) x {passes} row pass(es)",
-        "row_passes": passes, "groups": groups, "algorithmic_bytes_per_worker_coord": per_wc,
-        "moved_bytes_per_worker_coord": moved_wc,
-        "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-        "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
-        "frac_of_nominal_8000_GBps": round(k1_gbs / 8000.0, 4),
-        "traffic": k1_traffic_per_launch(w.name) if variant != "sketched_state" and groups * passes == 1 else None,
-        "algorithmic_bytes_per_launch": phase_bytes / (groups * passes) if passes == 1 else None,
-        "algorithmic_bytes_per_phase": phase_bytes,
-        "avg_launch_ms": round(sum(k1_ms) / len(k1_ms) / (groups * passes), 4),
-        "avg_phase_ms": round(sum(k1_ms) / len(k1_ms), 4),
-        "timed_phases": len(k1_ms),
-        "timing": "event-record nodes inside the step's CUDA graph" if use_plan else "CUDA events around the call",
-        "co_bound": {"kind": "SM->L2 payload: cell reductions (4*r B per worker-coordinate) + u, e stores "
-                             "(8 B per worker-coordinate; none for the sketched state)",
-                     "cell_updates_per_phase": cells,
-                     "achieved_G_cells_per_s": round(cells / phase_s / 1e9, 1),
-                     "probe_peak_G_cells_per_s": 134.5,
-                     "sm_to_l2_payload_GBps": round(P * d * (4 * r + (0 if variant == "sketched_state" else 8))
-                                                    / phase_s / 1e9, 1)},
-        "step_share": round(sum(k1_ms) / elapsed_ms, 3),
-    }
+    stream = torch.cuda.current_stream()
+    w = workloads.get_config(args.config)
+    if args.d:
+        w = shrink(w, args.d)
+        args.profile_steps = True
+    variant = args.variant
+    quick = args.profile_steps
 
-    # end to end through the public API with host buffers: a host plan per gradient set (the
-    # uploads where needed, the step and the download of idx and vals are one graph), then a
-    # stream synchronisation so that the host can read the step's result
+    sampler = None if quick else ClockSampler(gpu_uuid(dev))
+    if sampler:
+        sampler.start()
+    res, run = measure(gs, w, variant, args.eager, args.steps, args.warmup, world, rank, dev, stream, peaks,
+                       peak_kind, sampler, want_e2e=not (args.no_e2e or quick), probes=not quick)
+    clocks = sampler.stop() if sampler else None
+
     e2e = None
-    if not args.no_e2e and not args.profile_steps and variant == "error_feedback":
-        grad_dev = [torch.empty(d, dtype=torch.float32, device=dev) for _ in range(P)]
-        idx_h = torch.empty(k, dtype=torch.int64).pin_memory()
-        vals_h = torch.empty(k, dtype=torch.float32).pin_memory()
-        hplans = []
-        if use_plan:
-            hplans = [gs.gs_step_host_plan_create(sk, us, es, hb, grad_dev, d, rho, k, idx_h, vals_h, ws)
-                      for hb in host_pool]
+    if not args.no_e2e and not quick and variant == "error_feedback" and not run.streamed:
+        e2e = e2e_measure(gs, run, args.steps, args.warmup, world, dev)
+    W, groups = run.W, run.groups
+    run.close()
+    del run
+    torch.cuda.empty_cache()
 
-        def host_step(t):
-            if use_plan:
-                gs.gs_plan_launch(hplans[t % len(hplans)], stream)
-                stream.synchronize()
-            else:
-                gs.gs_step_host(sk, us, es, host_pool[t % len(host_pool)], grad_dev, d, rho, k, idx_h, vals_h, ws,
-                                None, stream)
-
-        for t in range(max(args.warmup, len(hplans))):  # every plan once, at least W steps
-            host_step(t)
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for t in range(args.steps):
-            host_step(args.warmup + t)
-        torch.cuda.synchronize()
-        e2e_s = time.perf_counter() - t0
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
-        e2e_s = dist_max(e2e_s, dev)
-        for hp in hplans:
-            gs.gs_plan_destroy(hp)
-        e2e = {"value": whole_job_rate(world, P, d, args.steps, e2e_s), "unit": UNIT, "h2d_bytes_per_step": P * d * 4,
-               "d2h_bytes_per_step": k * (8 + 4), "ms_per_step": round(e2e_s * 1e3 / args.steps, 4),
-               "call": "gs_step_host_plan_create + gs_plan_launch" if use_plan else "gs_step_host"}
-
-    for plan in plans:
-        gs.gs_plan_destroy(plan)
+    per_config = None
+    if not args.no_per_config and not quick and variant == "error_feedback":
+        per_config = {}
+        for name in sorted(workloads.CONFIGS, key=lambda n: workloads.CONFIGS[n].d):
+            wc = workloads.get_config(name)
+            if name == w.name:
+                per_config[name] = short_summary(res, wc)
+                continue
+            steps = PER_CONFIG_STEPS.get(name, 5)
+            rc, runc = measure(gs, wc, variant, args.eager, steps, max(3, min(args.warmup, 5)), world, rank, dev,
+                               stream, peaks, peak_kind)
+            per_config[name] = short_summary(rc, wc)
+            runc.close()
+            del runc
+            torch.cuda.empty_cache()
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_steps \
-            and variant == "error_feedback":
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not quick and variant == "error_feedback":
         cpu = cpu_baseline(w, steps=2)
 
-    gs.gs_sketch_destroy(sk)
-    for extra in (sk_u, sk_e):
-        if extra:
-            gs.gs_sketch_destroy(extra)
-    # insert (one per group and row pass), merge, query + selection (7; HEAVYMIX 10), then
-    # the gather (sketched state: cell accumulate, take, query_at, two sparse inserts, update)
-    # the top-k query adds its repair check where it prunes rows (d >= 2^22, r >= 3, c a power of two)
-    prunes = variant != "heavymix" and d >= (1 << 22) and r >= 3 and (c & (c - 1)) == 0
-    launches_per_step = groups * passes + 1 + (10 if variant == "heavymix" else 7) + (1 if prunes else 0) + \
-        (6 if variant == "sketched_state" else 1)
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 4), "higher_is_better": True,
+        "metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": w.name, "variant": variant, "launch": "plan" if use_plan else "eager",
-                   "warmup_steps_run": n_warm, "d": d, "P": P, "r": r, "c": c, "k": k, "rho": rho, "group_width": W,
+        "config": {"workload": w.name, "variant": variant, "launch": res["launch"],
+                   "warmup_steps_run": res["warmup_steps_run"], "d": w.d, "P": w.P, "r": w.r, "c": w.c, "k": w.k,
+                   "rho": w.rho, "group_width": W, "groups": groups,
                    "parallelism": f"replicas{world}" if world > 1 else "single-gpu",
-                   "l2": f"inputs larger than L2 ({P * d * 12 / 1e9:.2f} GB of g,u,e streamed per step)",
-                   "d_steps_per_s": world * d * args.steps / (elapsed_ms / 1e3)},
-        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
-        "clocks": clocks,
+                   "l2": res["l2"], "d_steps_per_s": world * w.d * args.steps / (res["ms_per_step"] * args.steps / 1e3)},
+        "roofline": res["roofline"], "roofline_query": res["roofline_query"], "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": res["gpu_launches_per_step"] * args.steps, "clocks": clocks,
+        "insert_share_of_step": res["insert_share_of_step"],
     }
+    for key in ("streaming", "ms_per_step_without_generation", "query_and_selection_ms"):
+        if key in res:
+            line[key] = res[key]
+    if per_config is not None:
+        line["per_config"] = per_config
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -124,6 +124,20 @@ gs_status gs_accumulate_insert(gs_sketch* sketch, int32_t first_worker, int32_t 
                                const float* const* grad, int64_t d, float rho,
                                gs_stream stream);
 
+/* gs_accumulate_insert with the cell updates staged in shared memory: gs_accumulate for each
+ * worker of the range, then one kernel per group in which every CTA holds one table row of up
+ * to four of the group's workers in shared memory ([c][workers] fp32), adds a contiguous chunk
+ * of the coordinates into it with shared-memory atomic additions, and flushes the tile into
+ * the table with one vector reduction per touched bucket.  Same arguments, constraints and
+ * result as gs_accumulate_insert (up to the order of the fp32 additions), but only for
+ * sketches whose row of c cells fits a tile: c * 4 bytes <= 200 KiB (GS_ERR_INVALID_ARG
+ * otherwise).  On GB300 it is slower than the direct reductions of gs_accumulate_insert at
+ * every size where it applies; the library's steps use gs_accumulate_insert. */
+gs_status gs_accumulate_insert_staged(gs_sketch* sketch, int32_t first_worker, int32_t n_workers,
+                                      float* const* momentum, float* const* error,
+                                      const float* const* grad, int64_t d, float rho,
+                                      gs_stream stream);
+
 /* ---- step 3: tree merge ---------------------------------------------------------- */
 
 /* Merge the tables of workers 0..P-1 into the merged table by recursive halving
@@ -250,6 +264,19 @@ gs_status gs_train_step(gs_sketch* sketch, float* weights, float lr, float* cons
                         int64_t k, int64_t* idx_out, float* vals_out, float* est_out,
                         void* workspace, size_t workspace_bytes, gs_stream stream);
 
+/* Device workspace bytes gs_heavymix_step needs. */
+gs_status gs_heavymix_step_workspace_size(int64_t d, int64_t k, size_t* bytes);
+
+/* gs_step with the HEAVYMIX selection of gs_query_heavymix (Alg. 2 steps 1-3 as printed, with
+ * the fill drawn from fill_seed) in place of the deterministic top-k: gs_sketch_zero,
+ * gs_accumulate_insert, gs_sketch_merge_tree, gs_query_heavymix (its estimate kept in the
+ * workspace; l2sq_out, one device double, may be NULL), gs_gather_and_zero.  workspace:
+ * gs_heavymix_step_workspace_size(d, k) bytes, 256-byte aligned. */
+gs_status gs_heavymix_step(gs_sketch* sketch, float* const* momentum, float* const* error,
+                           const float* const* grad, int64_t d, float rho, int64_t k,
+                           uint64_t fill_seed, int64_t* idx_out, float* vals_out, double* l2sq_out,
+                           void* workspace, size_t workspace_bytes, gs_stream stream);
+
 /* ---- momentum and error kept as sketches ------------------------------------------ */
 /* Sec. II notes that a linear sketch can carry momentum and error accumulation itself.  In
  * this variant the state is two r x c tables instead of 2P vectors of length d: the
@@ -311,15 +338,18 @@ gs_status gs_step_host(gs_sketch* sketch, float* const* momentum, float* const* 
  * are reused as in the direct calls.  All of them must stay allocated until
  * gs_plan_destroy.  The sketches must not be destroyed first.  A plan is not thread-safe.
  *
- * flags: 0, or GS_PLAN_TIME_INSERT to bracket the insert phase (zeroed tables excluded) with
- * two event-record nodes; launch n records into slot n mod 1024 of a ring of event pairs, and
- * gs_plan_insert_times reads them.
+ * flags: 0, or any of GS_PLAN_TIME_INSERT, which brackets the insert phase (zeroed tables
+ * excluded) with two event-record nodes, and GS_PLAN_TIME_QUERY, which records three: before
+ * the median query (after its workspace is cleared), after it (its prune-key sample and repair
+ * check included) and after the top-k selection.  Launch n records into slot n mod 1024 of a
+ * ring of events per node; gs_plan_insert_times and gs_plan_query_times read them.
  *
  * Errors: the same argument checks as the direct call (GS_ERR_INVALID_ARG, GS_ERR_MISMATCH);
  * GS_ERR_CUDA if capture or instantiation fails (for example a host gradient that is neither
  * device-addressable nor pinned, whose upload cannot be captured).  Nothing is launched while
  * a plan is created. */
 #define GS_PLAN_TIME_INSERT 1
+#define GS_PLAN_TIME_QUERY 2
 
 /* gs_step (weights == NULL) or gs_train_step (weights != NULL, with lr) as a plan. */
 gs_status gs_step_plan_create(gs_sketch* sketch, float* const* momentum, float* const* error,
@@ -327,6 +357,13 @@ gs_status gs_step_plan_create(gs_sketch* sketch, float* const* momentum, float* 
                               int64_t* idx_out, float* vals_out, float* est_out, float* weights,
                               float lr, void* workspace, size_t workspace_bytes, int32_t flags,
                               gs_plan** plan_out);
+
+/* gs_heavymix_step as a plan. */
+gs_status gs_heavymix_step_plan_create(gs_sketch* sketch, float* const* momentum, float* const* error,
+                                       const float* const* grad, int64_t d, float rho, int64_t k,
+                                       uint64_t fill_seed, int64_t* idx_out, float* vals_out,
+                                       double* l2sq_out, void* workspace, size_t workspace_bytes,
+                                       int32_t flags, gs_plan** plan_out);
 
 /* gs_step_host as a plan.  The uploads (where needed) and the download of idx and vals into
  * idx_host / vals_host are part of the graph; a launch does NOT synchronise: synchronise the
@@ -352,8 +389,47 @@ gs_status gs_plan_launch(gs_plan* plan, gs_stream stream);
  * GS_ERR_INVALID_ARG if the plan was created without GS_PLAN_TIME_INSERT. */
 gs_status gs_plan_insert_times(gs_plan* plan, float* ms_out, int32_t n, int32_t* n_out);
 
+/* Median-query and selection durations in ms of the last min(n, launches, 1024) launches,
+ * oldest first: query_ms_out[t] from before the query to after its repair check (steps 4),
+ * select_ms_out[t] from there to after the top-k selection (steps 5), both HOST arrays of n
+ * floats; *n_out = how many.  Waits for the last launch to finish.  GS_ERR_INVALID_ARG if the
+ * plan was created without GS_PLAN_TIME_QUERY. */
+gs_status gs_plan_query_times(gs_plan* plan, float* query_ms_out, float* select_ms_out, int32_t n,
+                              int32_t* n_out);
+
 /* Wait for the device to go idle if the plan was ever launched, then free it.  NULL is OK. */
 gs_status gs_plan_destroy(gs_plan* plan);
+
+/* ---- measurement aid --------------------------------------------------------------- */
+/* The fused insert (gs_accumulate_insert over every group and row pass) is bound by the
+ * requests its SMs send to L2: one cell reduction per (coordinate, row, group) and the
+ * momentum and error stores, rather than by HBM bandwidth.  gs_insert_request_ceiling
+ * measures the time of that request mix with HBM taken out: it runs the insert kernels of one
+ * whole insert phase for d coordinates and all of the sketch's workers, with the same grids,
+ * instructions, hash buckets and cell reductions, but with every vector access folded into an
+ * L2-resident window (GS_CEILING_WINDOW_FLOATS floats per vector).  Not a step of the method
+ * (the paper has no counterpart); it only gives the insert's roofline a measured second
+ * bound.  window: a device buffer of gs_insert_request_ceiling_window_size bytes, 256-byte
+ * aligned, overwritten.  The worker tables are left unspecified: zero them before the next
+ * insert.  *ms_out (host) receives the elapsed time of the phase, measured with events on
+ * `stream`; the call synchronizes with them.  GS_ERR_INVALID_ARG unless the group width is
+ * 4, 8 or 16 and c is a power of two. */
+#define GS_CEILING_WINDOW_FLOATS (1 << 17)
+
+gs_status gs_insert_request_ceiling_window_size(const gs_sketch* sketch, size_t* bytes);
+
+gs_status gs_insert_request_ceiling(gs_sketch* sketch, int64_t d, void* window, size_t window_bytes,
+                                    float* ms_out, gs_stream stream);
+
+/* The median query is bound by its r scattered 4-byte reads per coordinate from the merged
+ * table (each one a separate sector request from L1 to L2), not by HBM.  This probe runs the
+ * query kernel's loads alone for d coordinates (all r rows, the same grid and hash buckets,
+ * no median, no estimate store, no histogram), so that d*r requests over *ms_out (host) is a
+ * measured ceiling of that request stream.  window: at least 65536 bytes of device memory,
+ * 256-byte aligned, overwritten (one float per CTA).  The call synchronizes with its events.
+ * Not a step of the method.  GS_ERR_INVALID_ARG unless c is a power of two. */
+gs_status gs_query_request_ceiling(const gs_sketch* sketch, int64_t d, void* window, size_t window_bytes,
+                                   float* ms_out, gs_stream stream);
 
 /* ---- inspection hooks ------------------------------------------------------------ */
 

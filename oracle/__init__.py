@@ -42,8 +42,11 @@ from .gssgd import (  # noqa: F401
     query,
     cell_band,
     topk,
+    topk_by_threshold,
     heavymix,
     heavymix_select,
+    heavymix_members,
+    heavymix_select_from,
     gather_and_zero,
     apply_update,
     query_at,

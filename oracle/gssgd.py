@@ -58,16 +58,23 @@ def accumulate(u: np.ndarray, e: np.ndarray, g: np.ndarray, rho: float):
 
 # ---- 2. sketch -------------------------------------------------------------------------
 
-def sketch(x: np.ndarray, coeffs, c: int, hashes=None):
+def sketch(x: np.ndarray, coeffs, c: int, hashes=None, idx=None):
     """Count Sketch of vector x: (T, A), both [r, c] fp64.
 
     T[j][b] = sum over i with h_j(i) = b of s_j(i) * x_i
     A[j][b] = sum over the same i of |x_i|       (the magnitude carried by the cell)
-    ``hashes`` may pass ``hash_rows(coeffs, c, arange(d))`` computed once for many vectors.
+    ``idx`` gives the global coordinate of each entry of x (default 0 .. len(x) - 1), so that
+    a long vector can be sketched piece by piece: by the linearity of the Count Sketch
+    (Sec. III-A), the sketch of x is the sum of the sketches of its pieces, each piece hashed
+    at its own global coordinates.  ``hashes`` may pass ``hash_rows(coeffs, c, idx)`` computed
+    once for many vectors.
     """
     x64 = np.asarray(x, dtype=np.float32).astype(np.float64)
     d = x64.size
-    buckets, signs = hashes if hashes is not None else hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+    if hashes is None:
+        gi = np.arange(d, dtype=np.uint64) if idx is None else np.asarray(idx, dtype=np.uint64)
+        hashes = hash_rows(coeffs, c, gi)
+    buckets, signs = hashes
     r = buckets.shape[0]
     T = np.zeros((r, c), dtype=np.float64)
     A = np.zeros((r, c), dtype=np.float64)
@@ -114,15 +121,20 @@ def merge_tree(tables):
 
 # ---- 4. query --------------------------------------------------------------------------
 
-def query(T: np.ndarray, coeffs, d: int, hashes=None):
-    """est_i = median over rows j of s_j(i) * T[j][h_j(i)] for i < d (fp64).
+def query(T: np.ndarray, coeffs, d: int, hashes=None, idx=None):
+    """est_i = median over rows j of s_j(i) * T[j][h_j(i)] for i < d (fp64), or for the global
+    coordinates ``idx`` when given (then d = len(idx)).
 
     With an odd number of rows the median is the middle order statistic; with an even
     number it is the mean of the two middle ones.
     """
     c = T.shape[1]
-    buckets, signs = hashes if hashes is not None else hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+    if hashes is None:
+        gi = np.arange(d, dtype=np.uint64) if idx is None else np.asarray(idx, dtype=np.uint64)
+        hashes = hash_rows(coeffs, c, gi)
+    buckets, signs = hashes
     r = buckets.shape[0]
+    d = buckets.shape[1]
     vals = np.empty((r, d), dtype=np.float64)
     for j in range(r):
         vals[j] = signs[j] * T[j][buckets[j]]
@@ -132,10 +144,11 @@ def query(T: np.ndarray, coeffs, d: int, hashes=None):
     return 0.5 * (vals[r // 2 - 1] + vals[r // 2])
 
 
-def cell_band(A: np.ndarray, coeffs, idx, rel: float = 1e-5):
-    """Per-coordinate tolerance band rel * max_j A[j][h_j(i)] for the median estimate."""
+def cell_band(A: np.ndarray, coeffs, idx, rel: float = 1e-5, hashes=None):
+    """Per-coordinate tolerance band rel * max_j A[j][h_j(i)] for the median estimate, at the
+    coordinates idx (or at those whose ``hash_rows`` are passed as ``hashes``)."""
     c = A.shape[1]
-    buckets, _ = hash_rows(coeffs, c, np.asarray(idx, dtype=np.uint64))
+    buckets, _ = hashes if hashes is not None else hash_rows(coeffs, c, np.asarray(idx, dtype=np.uint64))
     r = buckets.shape[0]
     mags = np.stack([A[j][buckets[j]] for j in range(r)])
     return rel * mags.max(axis=0)
@@ -150,17 +163,41 @@ def topk(est: np.ndarray, k: int) -> np.ndarray:
     return np.sort(order[:k]).astype(np.int64)
 
 
+def topk_by_threshold(est: np.ndarray, k: int) -> np.ndarray:
+    """The same set as ``topk``, found without a full sort (for vectors of hundreds of millions
+    of entries): tau = the k-th largest |est|; every index with |est| > tau, then the
+    k - #{|est| > tau} smallest indices with |est| == tau; ascending."""
+    a = np.abs(np.asarray(est, dtype=np.float64))
+    tau = np.partition(a, a.size - k)[a.size - k]
+    gt = np.nonzero(a > tau)[0]
+    eq = np.nonzero(a == tau)[0]
+    return np.sort(np.concatenate([gt, eq[: k - gt.size]])).astype(np.int64)
+
+
 # ---- 5'. HEAVYMIX ----------------------------------------------------------------------
 
 def heavymix_select(est: np.ndarray, l2sq: float, k: int, fill_seed: int) -> np.ndarray:
     """Alg. 2 steps 2-3 from given estimates and ||g||^2 estimate (indices ascending):
-    H = {i : est_i^2 >= l2sq / k}, est_i taken at fp32 precision and squared exactly; if
+    H = {i : est_i^2 >= l2sq / k}, evaluated in fp64 on the estimates as given; if
     |H| >= k the k members of H with largest |est| (ties to the smaller index), else H plus the
     l = k - |H| members of NH with the smallest xi_i = splitmix64_at(fill_seed, i) >> 33,
     ties to the smaller index (a uniformly random l-subset of NH)."""
     est = np.asarray(est, dtype=np.float64)
-    est32 = est.astype(np.float32).astype(np.float64)
-    in_h = est32 * est32 >= l2sq / k
+    in_h = heavymix_members(est, l2sq, k)
+    return heavymix_select_from(in_h, est, k, fill_seed)
+
+
+def heavymix_members(est: np.ndarray, l2sq: float, k: int) -> np.ndarray:
+    """The membership mask of H = {i : est_i^2 >= l2sq / k} (Alg. 2 step 2), in fp64."""
+    est = np.asarray(est, dtype=np.float64)
+    return est * est >= l2sq / k
+
+
+def heavymix_select_from(in_h: np.ndarray, est: np.ndarray, k: int, fill_seed: int) -> np.ndarray:
+    """Alg. 2 step 3 for a given membership mask of H: the top-k of H by |est| when |H| >= k,
+    else H plus the first k - |H| members of NH in the fill order (xi_i, i)."""
+    est = np.asarray(est, dtype=np.float64)
+    in_h = np.asarray(in_h, dtype=bool)
     nh = int(in_h.sum())
     if nh >= k:
         return topk(np.where(in_h, est, 0.0), k)

@@ -25,6 +25,7 @@ GS_MAX_COLS = 1 << 26
 GS_MAX_WORKERS = 64
 GS_MAX_DIM = (1 << 31) - 1
 GS_NOALLOC_MAX_DIM = 1 << 30
+GS_CEILING_WINDOW_FLOATS = 1 << 17
 
 _lib = None
 
@@ -43,6 +44,7 @@ SIGNATURES = {
     "gs_accumulate": [_vp, _vp, _vp, _i64, _f32, _vp],
     "gs_sketch_insert": [_vp, _i32, _vp, _i64, _vp],
     "gs_accumulate_insert": [_vp, _i32, _i32, _PP, _PP, _PP, _i64, _f32, _vp],
+    "gs_accumulate_insert_staged": [_vp, _i32, _i32, _PP, _PP, _PP, _i64, _f32, _vp],
     "gs_sketch_merge_tree": [_vp, _i32, _vp],
     "gs_query_topk_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_query_topk": [_vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp],
@@ -53,6 +55,10 @@ SIGNATURES = {
     "gs_apply_update": [_vp, _i64, _vp, _vp, _i64, _f32, _vp],
     "gs_gather_zero_update": [_PP, _PP, _i32, _i64, _vp, _i64, _vp, _vp, _f32, _vp],
     "gs_train_step": [_vp, _vp, _f32, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
+    "gs_heavymix_step_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
+    "gs_heavymix_step": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _u64, _vp, _vp, _vp, _vp, _sz, _vp],
+    "gs_heavymix_step_plan_create": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _u64, _vp, _vp, _vp, _vp, _sz, _i32,
+                                     ctypes.POINTER(_vp)],
     "gs_sketch_merged_table": [_vp, ctypes.POINTER(_vp)],
     "gs_sketch_query_at": [_vp, _vp, _i64, _vp, _vp],
     "gs_sketch_add_sparse": [_vp, _vp, _vp, _i64, _f32, _vp],
@@ -65,10 +71,14 @@ SIGNATURES = {
                                       ctypes.POINTER(_vp)],
     "gs_plan_launch": [_vp, _vp],
     "gs_plan_insert_times": [_vp, _vp, _i32, ctypes.POINTER(_i32)],
+    "gs_plan_query_times": [_vp, _vp, _vp, _i32, ctypes.POINTER(_i32)],
     "gs_plan_destroy": [_vp],
     "gs_step_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_step": [_vp, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _vp, _sz, _vp],
     "gs_step_host": [_vp, _PP, _PP, _PP, _PP, _i64, _f32, _i64, _vp, _vp, _vp, _sz, _vp],
+    "gs_insert_request_ceiling_window_size": [_vp, ctypes.POINTER(_sz)],
+    "gs_insert_request_ceiling": [_vp, _i64, _vp, _sz, ctypes.POINTER(_f32), _vp],
+    "gs_query_request_ceiling": [_vp, _i64, _vp, _sz, ctypes.POINTER(_f32), _vp],
     "gs_hash_eval": [_vp, _vp, _i64, _vp, _vp, _vp],
     "gs_sketch_copy_to_host": [_vp, _i32, _vp],
     "gs_last_error": [],
@@ -174,6 +184,14 @@ def gs_accumulate_insert(sketch: int, first_worker: int, momentum, error, grad, 
     _check(load_library().gs_accumulate_insert(sketch, first_worker, n, _ptr_array(momentum),
                                                _ptr_array(error), _ptr_array(grad), d, rho,
                                                _stream(stream)), "gs_accumulate_insert")
+
+
+def gs_accumulate_insert_staged(sketch: int, first_worker: int, momentum, error, grad, d: int,
+                                rho: float, stream=None) -> None:
+    n = len(grad)
+    _check(load_library().gs_accumulate_insert_staged(sketch, first_worker, n, _ptr_array(momentum),
+                                                      _ptr_array(error), _ptr_array(grad), d, rho,
+                                                      _stream(stream)), "gs_accumulate_insert_staged")
 
 
 def gs_sketch_merge_tree(sketch: int, P: int, stream=None) -> None:
@@ -295,10 +313,36 @@ def gs_step_host(sketch: int, momentum, error, grad_host, grad_dev, d: int, rho:
 
 
 GS_PLAN_TIME_INSERT = 1
+GS_PLAN_TIME_QUERY = 2
 
 
 def _nbytes(workspace, workspace_bytes):
     return workspace.numel() * workspace.element_size() if workspace_bytes is None else workspace_bytes
+
+
+def gs_heavymix_step_workspace_size(d: int, k: int) -> int:
+    out = _sz()
+    _check(load_library().gs_heavymix_step_workspace_size(d, k, ctypes.byref(out)), "gs_heavymix_step_workspace_size")
+    return out.value
+
+
+def gs_heavymix_step(sketch: int, momentum, error, grad, d: int, rho: float, k: int, fill_seed: int, idx_out,
+                     vals_out, l2sq_out, workspace, workspace_bytes=None, stream=None) -> None:
+    _check(load_library().gs_heavymix_step(sketch, _ptr_array(momentum), _ptr_array(error), _ptr_array(grad), d, rho,
+                                           k, fill_seed, _ptr(idx_out), _ptr(vals_out), _ptr(l2sq_out),
+                                           _ptr(workspace), _nbytes(workspace, workspace_bytes), _stream(stream)),
+           "gs_heavymix_step")
+
+
+def gs_heavymix_step_plan_create(sketch: int, momentum, error, grad, d: int, rho: float, k: int, fill_seed: int,
+                                 idx_out, vals_out, l2sq_out, workspace, workspace_bytes=None, flags: int = 0) -> int:
+    out = _vp()
+    _check(load_library().gs_heavymix_step_plan_create(sketch, _ptr_array(momentum), _ptr_array(error),
+                                                       _ptr_array(grad), d, rho, k, fill_seed, _ptr(idx_out),
+                                                       _ptr(vals_out), _ptr(l2sq_out), _ptr(workspace),
+                                                       _nbytes(workspace, workspace_bytes), flags,
+                                                       ctypes.byref(out)), "gs_heavymix_step_plan_create")
+    return out.value
 
 
 def gs_step_plan_create(sketch: int, momentum, error, grad, d: int, rho: float, k: int, idx_out, vals_out,
@@ -346,8 +390,41 @@ def gs_plan_insert_times(plan: int, n: int = 1024) -> list:
     return [float(buf[i]) for i in range(got.value)]
 
 
+def gs_plan_query_times(plan: int, n: int = 1024) -> tuple:
+    """(query_ms, select_ms): lists over the last launches, oldest first."""
+    q = (ctypes.c_float * max(n, 1))()
+    sel = (ctypes.c_float * max(n, 1))()
+    got = _i32()
+    _check(load_library().gs_plan_query_times(plan, ctypes.cast(q, _vp), ctypes.cast(sel, _vp), n,
+                                              ctypes.byref(got)), "gs_plan_query_times")
+    return [float(q[i]) for i in range(got.value)], [float(sel[i]) for i in range(got.value)]
+
+
 def gs_plan_destroy(plan: int) -> None:
     _check(load_library().gs_plan_destroy(plan), "gs_plan_destroy")
+
+
+def gs_insert_request_ceiling_window_size(sketch: int) -> int:
+    out = _sz()
+    _check(load_library().gs_insert_request_ceiling_window_size(sketch, ctypes.byref(out)),
+           "gs_insert_request_ceiling_window_size")
+    return out.value
+
+
+def gs_insert_request_ceiling(sketch: int, d: int, window, window_bytes=None, stream=None) -> float:
+    """Milliseconds of one insert phase's request mix with the vectors held in L2."""
+    ms = _f32()
+    _check(load_library().gs_insert_request_ceiling(sketch, d, _ptr(window), _nbytes(window, window_bytes),
+                                                    ctypes.byref(ms), _stream(stream)), "gs_insert_request_ceiling")
+    return float(ms.value)
+
+
+def gs_query_request_ceiling(sketch: int, d: int, window, window_bytes=None, stream=None) -> float:
+    """Milliseconds of the median query's loads alone (all r rows) for d coordinates."""
+    ms = _f32()
+    _check(load_library().gs_query_request_ceiling(sketch, d, _ptr(window), _nbytes(window, window_bytes),
+                                                   ctypes.byref(ms), _stream(stream)), "gs_query_request_ceiling")
+    return float(ms.value)
 
 
 def gs_hash_eval(sketch: int, coords, n: int, bucket_out, sign_out, stream=None) -> None:

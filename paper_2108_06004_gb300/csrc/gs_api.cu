@@ -19,12 +19,17 @@ struct gs_sketch {
   int device;
 };
 
+// Events recorded between the phases of a step while it is captured into a plan, where each
+// becomes an event-record node of the graph: the insert phase, the query (sample, median
+// query and repair check) and the selection that follows it.
+enum PhaseMark { kInsertBegin, kInsertEnd, kQueryBegin, kQueryEnd, kSelectEnd, kMarks };
+
 struct gs_plan {
   cudaGraph_t graph = nullptr;
   cudaGraphExec_t exec = nullptr;
-  bool timed = false;
-  cudaGraphNode_t node_begin = nullptr, node_end = nullptr;  // event-record nodes around the insert phase
-  std::vector<cudaEvent_t> ev_begin, ev_end;                 // their ring of events
+  int32_t flags = 0;
+  cudaGraphNode_t node[kMarks] = {};     // the event-record nodes of the marks in use
+  std::vector<cudaEvent_t> ev[kMarks];   // their rings of events
   int64_t launches = 0;
   int device = 0;
 };
@@ -210,27 +215,34 @@ bool same_family(const gs_sketch* a, const gs_sketch* b) {
   return a->r == b->r && a->c == b->c && a->seed == b->seed;
 }
 
-// Optional events recorded around the insert phase of a step.  They are used only while a
-// step is captured into a plan, where each becomes an event-record node of the graph.
+// Optional events recorded between the phases of a step (unset entries record nothing).  They
+// are used only while a step is captured into a plan.
 struct InsertMarks {
-  cudaEvent_t begin = nullptr, end = nullptr;
+  cudaEvent_t ev[kMarks] = {};
 };
 
 cudaError_t mark(cudaEvent_t ev, cudaStream_t s) {
   return ev ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal) : cudaSuccess;
 }
 
+// The selection of a step: the deterministic top-k (default), or HEAVYMIX (Alg. 2 as printed).
+struct Selection {
+  bool heavymix = false;
+  uint64_t fill_seed = 0;
+  double* l2sq_out = nullptr;
+};
+
 gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float* const* g,
                     int64_t d, float rho, int64_t k, int64_t* idx, float* vals, float* est,
                     void* ws, cudaStream_t s, float* weights = nullptr, float lr = 0.f,
-                    InsertMarks marks = InsertMarks()) {
+                    InsertMarks marks = InsertMarks(), Selection sel = Selection()) {
   const size_t bytes = (size_t)sk->groups * sk->r * sk->c * sk->W * sizeof(float) +
                        (size_t)sk->r * sk->c * sizeof(float);
   cudaError_t err = cudaMemsetAsync(sk->tables, 0, bytes, s);
   if (err != cudaSuccess) return cuda_fail(err, "zero tables");
-  if ((err = mark(marks.begin, s)) != cudaSuccess) return cuda_fail(err, "event record");
+  if ((err = mark(marks.ev[kInsertBegin], s)) != cudaSuccess) return cuda_fail(err, "event record");
   GS_TRY(accumulate_insert_impl(sk, 0, sk->workers, m, e, g, d, rho, s));
-  if ((err = mark(marks.end, s)) != cudaSuccess) return cuda_fail(err, "event record");
+  if ((err = mark(marks.ev[kInsertEnd], s)) != cudaSuccess) return cuda_fail(err, "event record");
   gs::MergeParams mp;
   mp.tables = sk->tables;
   mp.merged = sk->merged;
@@ -238,9 +250,14 @@ gs_status step_impl(gs_sketch* sk, float* const* m, float* const* e, const float
   mp.group_stride = (int64_t)sk->r * sk->c * sk->W;
   mp.P = sk->workers;
   if ((err = gs::launch_merge(mp, sk->W, s)) != cudaSuccess) return cuda_fail(err, "merge launch");
-  if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, s)) !=
-      cudaSuccess)
+  if (sel.heavymix) {
+    if ((err = gs::launch_query_heavymix(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, sel.fill_seed, idx, est,
+                                         sel.l2sq_out, ws, s, &marks.ev[kQueryBegin])) != cudaSuccess)
+      return cuda_fail(err, "HEAVYMIX query launch");
+  } else if ((err = gs::launch_query_topk(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, k, idx, est, ws, s,
+                                          &marks.ev[kQueryBegin])) != cudaSuccess) {
     return cuda_fail(err, "query/top-k launch");
+  }
   gs::GatherParams gp;
   std::memset(&gp, 0, sizeof(gp));
   for (int p = 0; p < sk->workers; ++p) {
@@ -305,9 +322,9 @@ gs_status sketched_state_impl(gs_sketch* workers, gs_sketch* momentum, gs_sketch
   const size_t tbytes = ((size_t)workers->groups * workers->r * workers->c * workers->W + (size_t)cells) * sizeof(float);
   cudaError_t err = cudaMemsetAsync(workers->tables, 0, tbytes, s);
   if (err != cudaSuccess) return cuda_fail(err, "zero tables");
-  if ((err = mark(marks.begin, s)) != cudaSuccess) return cuda_fail(err, "event record");
+  if ((err = mark(marks.ev[kInsertBegin], s)) != cudaSuccess) return cuda_fail(err, "event record");
   GS_TRY(insert_all_impl(workers, grad, d, s));
-  if ((err = mark(marks.end, s)) != cudaSuccess) return cuda_fail(err, "event record");
+  if ((err = mark(marks.ev[kInsertEnd], s)) != cudaSuccess) return cuda_fail(err, "event record");
   gs::MergeParams mp;
   mp.tables = workers->tables;
   mp.merged = workers->merged;
@@ -320,7 +337,7 @@ gs_status sketched_state_impl(gs_sketch* workers, gs_sketch* momentum, gs_sketch
     return cuda_fail(err, "sketch accumulate launch");
   // top-k of the estimate from E; delta = that estimate at the selected coordinates
   if ((err = gs::launch_query_topk(error->merged, error->h, error->r, (uint32_t)error->c, d, k, idx, nullptr,
-                                   ws, s)) != cudaSuccess)
+                                   ws, s, &marks.ev[kQueryBegin])) != cudaSuccess)
     return cuda_fail(err, "query/top-k launch");
   const float* est = static_cast<const float*>(ws);  // the query keeps est at the ws start
   if ((err = gs::launch_take(est, d, idx, k, vals, s)) != cudaSuccess) return cuda_fail(err, "take launch");
@@ -425,10 +442,9 @@ constexpr int64_t kPlanRing = 1024;
 void plan_free(gs_plan* p) {
   if (p->exec) cudaGraphExecDestroy(p->exec);
   if (p->graph) cudaGraphDestroy(p->graph);
-  for (cudaEvent_t ev : p->ev_begin)
-    if (ev) cudaEventDestroy(ev);
-  for (cudaEvent_t ev : p->ev_end)
-    if (ev) cudaEventDestroy(ev);
+  for (int m = 0; m < kMarks; ++m)
+    for (cudaEvent_t ev : p->ev[m])
+      if (ev) cudaEventDestroy(ev);
   delete p;
 }
 
@@ -441,28 +457,33 @@ gs_status check_plan(const gs_plan* plan) {
   return GS_OK;
 }
 
-// Capture body(stream, marks) on a private stream into a graph and instantiate it.  With
-// GS_PLAN_TIME_INSERT the insert phase is bracketed by two event-record nodes whose events
-// each launch re-points into the ring.
+// The marks each plan flag records.
+bool mark_in_use(int32_t flags, int m) {
+  if (m == kInsertBegin || m == kInsertEnd) return (flags & GS_PLAN_TIME_INSERT) != 0;
+  return (flags & GS_PLAN_TIME_QUERY) != 0;
+}
+
+// Capture body(stream, marks) on a private stream into a graph and instantiate it.  Every
+// mark that the flags ask for becomes an event-record node whose event each launch re-points
+// into the mark's ring.
 template <class Body>
 gs_status capture_plan(int device, int32_t flags, gs_plan** out, Body&& body) {
   if (!out) return fail(GS_ERR_INVALID_ARG, "plan_out is NULL");
-  if (flags & ~int32_t(GS_PLAN_TIME_INSERT)) return fail(GS_ERR_INVALID_ARG, "unknown plan flags");
+  if (flags & ~int32_t(GS_PLAN_TIME_INSERT | GS_PLAN_TIME_QUERY)) return fail(GS_ERR_INVALID_ARG, "unknown plan flags");
   gs_plan* p = new gs_plan();
   p->device = device;
-  p->timed = (flags & GS_PLAN_TIME_INSERT) != 0;
+  p->flags = flags;
   cudaError_t e = cudaSuccess;
-  if (p->timed) {
-    p->ev_begin.assign((size_t)kPlanRing, nullptr);
-    p->ev_end.assign((size_t)kPlanRing, nullptr);
-    for (size_t i = 0; i < (size_t)kPlanRing && e == cudaSuccess; ++i) {
-      e = cudaEventCreate(&p->ev_begin[i]);
-      if (e == cudaSuccess) e = cudaEventCreate(&p->ev_end[i]);
-    }
-    if (e != cudaSuccess) {
-      plan_free(p);
-      return cuda_fail(e, "cudaEventCreate");
-    }
+  InsertMarks marks;
+  for (int m = 0; m < kMarks && e == cudaSuccess; ++m) {
+    if (!mark_in_use(flags, m)) continue;
+    p->ev[m].assign((size_t)kPlanRing, nullptr);
+    for (size_t i = 0; i < (size_t)kPlanRing && e == cudaSuccess; ++i) e = cudaEventCreate(&p->ev[m][i]);
+    marks.ev[m] = p->ev[m][0];
+  }
+  if (e != cudaSuccess) {
+    plan_free(p);
+    return cuda_fail(e, "cudaEventCreate");
   }
   cudaStream_t cs = nullptr;
   if ((e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking)) != cudaSuccess) {
@@ -474,11 +495,6 @@ gs_status capture_plan(int device, int32_t flags, gs_plan** out, Body&& body) {
     plan_free(p);
     return cuda_fail(e, "cudaStreamBeginCapture");
   }
-  InsertMarks marks;
-  if (p->timed) {
-    marks.begin = p->ev_begin[0];
-    marks.end = p->ev_end[0];
-  }
   const gs_status st = body(cs, marks);
   cudaGraph_t graph = nullptr;
   e = cudaStreamEndCapture(cs, &graph);
@@ -488,7 +504,7 @@ gs_status capture_plan(int device, int32_t flags, gs_plan** out, Body&& body) {
     plan_free(p);
     return st != GS_OK ? st : cuda_fail(e, "stream capture");
   }
-  if (p->timed) {
+  if (flags) {
     size_t n = 0;
     e = cudaGraphGetNodes(graph, nullptr, &n);
     std::vector<cudaGraphNode_t> nodes(n);
@@ -498,12 +514,15 @@ gs_status capture_plan(int device, int32_t flags, gs_plan** out, Body&& body) {
       if ((e = cudaGraphNodeGetType(nodes[i], &type)) != cudaSuccess || type != cudaGraphNodeTypeEventRecord) continue;
       cudaEvent_t ev = nullptr;
       if ((e = cudaGraphEventRecordNodeGetEvent(nodes[i], &ev)) != cudaSuccess) break;
-      if (ev == marks.begin) p->node_begin = nodes[i];
-      if (ev == marks.end) p->node_end = nodes[i];
+      for (int m = 0; m < kMarks; ++m)
+        if (ev && ev == marks.ev[m]) p->node[m] = nodes[i];
     }
-    if (e == cudaSuccess && (!p->node_begin || !p->node_end)) {
-      plan_free(p);
-      return fail(GS_ERR_CUDA, "stream capture: insert-phase event nodes not found");
+    for (int m = 0; m < kMarks && e == cudaSuccess; ++m) {
+      if (mark_in_use(flags, m) && !p->node[m]) {
+        cudaStreamDestroy(cs);
+        plan_free(p);
+        return fail(GS_ERR_CUDA, "stream capture: phase event nodes not found");
+      }
     }
   }
   if (e == cudaSuccess) e = cudaGraphInstantiate(&p->exec, graph, 0);
@@ -699,6 +718,51 @@ gs_status gs_accumulate_insert(gs_sketch* sk, int32_t first_worker, int32_t n_wo
   GS_GUARD_END
 }
 
+gs_status gs_accumulate_insert_staged(gs_sketch* sk, int32_t first_worker, int32_t n_workers, float* const* momentum,
+                                      float* const* error, const float* const* grad, int64_t d, float rho,
+                                      gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (n_workers < 1 || first_worker < 0 || first_worker + n_workers > sk->workers)
+    return fail(GS_ERR_INVALID_ARG, "worker range out of bounds");
+  if (first_worker % sk->W != 0) return fail(GS_ERR_INVALID_ARG, "first_worker must be a multiple of the group width");
+  const int end = first_worker + n_workers;
+  if (end % sk->W != 0 && end != sk->workers)
+    return fail(GS_ERR_INVALID_ARG, "the worker range must end on a group boundary or at the last worker");
+  if (!grad) return fail(GS_ERR_INVALID_ARG, "grad array is NULL");
+  GS_TRY(check_worker_arrays(n_workers, momentum, error, grad));
+  if (gs::staged_tile_width((uint32_t)sk->c, sk->W) == 0)
+    return fail(GS_ERR_INVALID_ARG, "a table row of c = " + std::to_string(sk->c) +
+                                        " cells does not fit a shared-memory tile (c * 4 bytes <= 200 KiB)");
+  cudaStream_t s = as_stream(stream);
+  for (int w = 0; w < n_workers; ++w) {
+    cudaError_t e = gs::launch_accumulate(momentum[w], error[w], grad[w], d, rho, s);
+    if (e != cudaSuccess) return cuda_fail(e, "accumulate launch");
+  }
+  const int W = sk->W;
+  for (int grp = first_worker / W; grp * W < end; ++grp) {
+    gs::InsertParams p;
+    std::memset(&p, 0, sizeof(p));
+    const int lo = grp * W;
+    const int nw = (end - lo) < W ? (end - lo) : W;
+    for (int w = 0; w < nw; ++w) p.e[w] = error[lo + w - first_worker];
+    p.table = sk->tables + (size_t)grp * sk->r * sk->c * W;
+    p.d = d;
+    p.nw = nw;
+    p.r = sk->r;
+    p.c = (uint32_t)sk->c;
+    p.cmask = (uint32_t)sk->c - 1;
+    p.h = sk->h;
+    p.j0 = 0;
+    p.j1 = sk->r;
+    cudaError_t e = gs::launch_insert_staged(p, W, s);
+    if (e != cudaSuccess) return cuda_fail(e, "staged insert launch");
+  }
+  return GS_OK;
+  GS_GUARD_END
+}
+
 gs_status gs_sketch_merge_tree(gs_sketch* sk, int32_t P, gs_stream stream) {
   GS_TRY(check_sketch(sk));
   if (P < 1 || P > sk->workers) return fail(GS_ERR_INVALID_ARG, "P must lie in [1, workers]");
@@ -880,6 +944,31 @@ gs_status gs_train_step(gs_sketch* sk, float* weights, float lr, float* const* m
   GS_GUARD_END
 }
 
+gs_status gs_heavymix_step_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_TRY(check_d(d));
+  if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
+  if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = gs::heavymix_workspace_bytes(d, k);
+  return GS_OK;
+}
+
+gs_status gs_heavymix_step(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad,
+                           int64_t d, float rho, int64_t k, uint64_t fill_seed, int64_t* idx_out, float* vals_out,
+                           double* l2sq_out, void* workspace, size_t workspace_bytes, gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_step(sk, momentum, error, grad, d, k, idx_out, vals_out, nullptr, workspace, workspace_bytes));
+  if (workspace_bytes < gs::heavymix_workspace_bytes(d, k))
+    return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_heavymix_step_workspace_size");
+  if (l2sq_out && !aligned(l2sq_out, 8)) return fail(GS_ERR_INVALID_ARG, "l2sq_out is not 8-byte aligned");
+  Selection sel;
+  sel.heavymix = true;
+  sel.fill_seed = fill_seed;
+  sel.l2sq_out = l2sq_out;
+  return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, nullptr, workspace, as_stream(stream),
+                   nullptr, 0.f, InsertMarks(), sel);
+  GS_GUARD_END
+}
+
 gs_status gs_sketch_merged_table(const gs_sketch* sk, float** table_out) {
   if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
   if (!table_out) return fail(GS_ERR_INVALID_ARG, "table_out is NULL");
@@ -953,6 +1042,27 @@ gs_status gs_step_plan_create(gs_sketch* sk, float* const* momentum, float* cons
   GS_GUARD_END
 }
 
+gs_status gs_heavymix_step_plan_create(gs_sketch* sk, float* const* momentum, float* const* error,
+                                      const float* const* grad, int64_t d, float rho, int64_t k, uint64_t fill_seed,
+                                      int64_t* idx_out, float* vals_out, double* l2sq_out, void* workspace,
+                                      size_t workspace_bytes, int32_t flags, gs_plan** plan_out) {
+  GS_GUARD_BEGIN
+  if (plan_out) *plan_out = nullptr;
+  GS_TRY(check_step(sk, momentum, error, grad, d, k, idx_out, vals_out, nullptr, workspace, workspace_bytes));
+  if (workspace_bytes < gs::heavymix_workspace_bytes(d, k))
+    return fail(GS_ERR_INVALID_ARG, "workspace too small: use gs_heavymix_step_workspace_size");
+  if (l2sq_out && !aligned(l2sq_out, 8)) return fail(GS_ERR_INVALID_ARG, "l2sq_out is not 8-byte aligned");
+  Selection sel;
+  sel.heavymix = true;
+  sel.fill_seed = fill_seed;
+  sel.l2sq_out = l2sq_out;
+  return capture_plan(sk->device, flags, plan_out, [&](cudaStream_t s, InsertMarks marks) {
+    return step_impl(sk, momentum, error, grad, d, rho, k, idx_out, vals_out, nullptr, workspace, s, nullptr, 0.f,
+                     marks, sel);
+  });
+  GS_GUARD_END
+}
+
 gs_status gs_step_host_plan_create(gs_sketch* sk, float* const* momentum, float* const* error,
                                    const float* const* grad_host, float* const* grad_dev, int64_t d, float rho,
                                    int64_t k, int64_t* idx_host, float* vals_host, void* workspace,
@@ -988,34 +1098,56 @@ gs_status gs_sketched_state_plan_create(gs_sketch* workers, gs_sketch* momentum,
 gs_status gs_plan_launch(gs_plan* plan, gs_stream stream) {
   GS_TRY(check_plan(plan));
   cudaError_t e = cudaSuccess;
-  if (plan->timed) {
-    const size_t slot = (size_t)(plan->launches % kPlanRing);
-    e = cudaGraphExecEventRecordNodeSetEvent(plan->exec, plan->node_begin, plan->ev_begin[slot]);
-    if (e == cudaSuccess) e = cudaGraphExecEventRecordNodeSetEvent(plan->exec, plan->node_end, plan->ev_end[slot]);
-    if (e != cudaSuccess) return cuda_fail(e, "plan event update");
-  }
+  const size_t slot = (size_t)(plan->launches % kPlanRing);
+  for (int m = 0; m < kMarks && e == cudaSuccess; ++m)
+    if (plan->node[m]) e = cudaGraphExecEventRecordNodeSetEvent(plan->exec, plan->node[m], plan->ev[m][slot]);
+  if (e != cudaSuccess) return cuda_fail(e, "plan event update");
   e = cudaGraphLaunch(plan->exec, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "cudaGraphLaunch");
   ++plan->launches;
   return GS_OK;
 }
 
-gs_status gs_plan_insert_times(gs_plan* plan, float* ms_out, int32_t n, int32_t* n_out) {
-  GS_TRY(check_plan(plan));
-  if (!plan->timed) return fail(GS_ERR_INVALID_ARG, "the plan was created without GS_PLAN_TIME_INSERT");
-  if (!ms_out || !n_out || n < 0) return fail(GS_ERR_INVALID_ARG, "ms_out or n_out is NULL, or n < 0");
+}  // extern "C"
+
+namespace {
+
+// Elapsed ms between marks a and b over the last min(n, launches, ring) launches, oldest first.
+gs_status plan_mark_times(gs_plan* plan, int a, int b, float* ms_out, int32_t n, int32_t* n_out) {
   int64_t m = n;
   if (m > plan->launches) m = plan->launches;
   if (m > kPlanRing) m = kPlanRing;
   *n_out = 0;
   if (m == 0) return GS_OK;
-  cudaError_t e = cudaEventSynchronize(plan->ev_end[(size_t)((plan->launches - 1) % kPlanRing)]);
+  cudaError_t e = cudaEventSynchronize(plan->ev[b][(size_t)((plan->launches - 1) % kPlanRing)]);
   for (int64_t t = 0; t < m && e == cudaSuccess; ++t) {
     const size_t slot = (size_t)((plan->launches - m + t) % kPlanRing);
-    e = cudaEventElapsedTime(&ms_out[t], plan->ev_begin[slot], plan->ev_end[slot]);
+    e = cudaEventElapsedTime(&ms_out[t], plan->ev[a][slot], plan->ev[b][slot]);
   }
   if (e != cudaSuccess) return cuda_fail(e, "plan event times");
   *n_out = (int32_t)m;
+  return GS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+gs_status gs_plan_insert_times(gs_plan* plan, float* ms_out, int32_t n, int32_t* n_out) {
+  GS_TRY(check_plan(plan));
+  if (!(plan->flags & GS_PLAN_TIME_INSERT)) return fail(GS_ERR_INVALID_ARG, "the plan was created without GS_PLAN_TIME_INSERT");
+  if (!ms_out || !n_out || n < 0) return fail(GS_ERR_INVALID_ARG, "ms_out or n_out is NULL, or n < 0");
+  return plan_mark_times(plan, kInsertBegin, kInsertEnd, ms_out, n, n_out);
+}
+
+gs_status gs_plan_query_times(gs_plan* plan, float* query_ms_out, float* select_ms_out, int32_t n, int32_t* n_out) {
+  GS_TRY(check_plan(plan));
+  if (!(plan->flags & GS_PLAN_TIME_QUERY)) return fail(GS_ERR_INVALID_ARG, "the plan was created without GS_PLAN_TIME_QUERY");
+  if (!query_ms_out || !select_ms_out || !n_out || n < 0)
+    return fail(GS_ERR_INVALID_ARG, "an output pointer is NULL, or n < 0");
+  int32_t n2 = 0;
+  GS_TRY(plan_mark_times(plan, kQueryBegin, kQueryEnd, query_ms_out, n, n_out));
+  GS_TRY(plan_mark_times(plan, kQueryEnd, kSelectEnd, select_ms_out, n, &n2));
   return GS_OK;
 }
 
@@ -1026,6 +1158,94 @@ gs_status gs_plan_destroy(gs_plan* plan) {
   plan_free(plan);
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
   return GS_OK;
+}
+
+gs_status gs_insert_request_ceiling_window_size(const gs_sketch* sk, size_t* bytes) {
+  GS_TRY(check_sketch(sk));
+  if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = (size_t)3 * sk->W * GS_CEILING_WINDOW_FLOATS * sizeof(float);
+  return GS_OK;
+}
+
+gs_status gs_insert_request_ceiling(gs_sketch* sk, int64_t d, void* window, size_t window_bytes, float* ms_out,
+                                    gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  const size_t need = (size_t)3 * sk->W * GS_CEILING_WINDOW_FLOATS * sizeof(float);
+  if (!window || !aligned(window, 256)) return fail(GS_ERR_INVALID_ARG, "window is NULL or not 256-byte aligned");
+  if (window_bytes < need) return fail(GS_ERR_INVALID_ARG, "window too small: need " + std::to_string(need));
+  if (!ms_out) return fail(GS_ERR_INVALID_ARG, "ms_out is NULL");
+  if (sk->W < 4 || (sk->c & (sk->c - 1)) != 0)
+    return fail(GS_ERR_INVALID_ARG, "the probe serves group widths 4, 8 and 16 with c a power of two");
+  cudaStream_t s = as_stream(stream);
+  cudaEvent_t ev[2] = {nullptr, nullptr};
+  cudaError_t e = cudaEventCreate(&ev[0]);
+  if (e == cudaSuccess) e = cudaEventCreate(&ev[1]);
+  // zero windows keep every value finite; the requests do not depend on the values
+  if (e == cudaSuccess) e = cudaMemsetAsync(window, 0, need, s);
+  if (e == cudaSuccess) e = cudaEventRecord(ev[0], s);
+  float* win = static_cast<float*>(window);
+  const int W = sk->W;
+  for (int grp = 0; e == cudaSuccess && grp * W < sk->workers; ++grp) {
+    gs::InsertParams p;
+    std::memset(&p, 0, sizeof(p));
+    const int nw = (sk->workers - grp * W) < W ? (sk->workers - grp * W) : W;
+    for (int w = 0; w < nw; ++w) {
+      p.u[w] = win + (size_t)(3 * w + 0) * GS_CEILING_WINDOW_FLOATS;
+      p.e[w] = win + (size_t)(3 * w + 1) * GS_CEILING_WINDOW_FLOATS;
+      p.g[w] = win + (size_t)(3 * w + 2) * GS_CEILING_WINDOW_FLOATS;
+    }
+    p.table = sk->tables + (size_t)grp * sk->r * sk->c * W;
+    p.d = d;
+    p.nw = nw;
+    p.r = sk->r;
+    p.c = (uint32_t)sk->c;
+    p.cmask = (uint32_t)sk->c - 1;
+    p.rho = 0.9f;
+    p.winmask = GS_CEILING_WINDOW_FLOATS - 1;
+    p.h = sk->h;
+    for (int j0 = 0; e == cudaSuccess && j0 < sk->r; j0 += sk->rows_per_pass) {
+      p.j0 = j0;
+      p.j1 = (j0 + sk->rows_per_pass < sk->r) ? j0 + sk->rows_per_pass : sk->r;
+      e = gs::launch_insert_ceiling_probe(p, W, j0 == 0, s);
+    }
+  }
+  if (e == cudaSuccess) e = cudaEventRecord(ev[1], s);
+  if (e == cudaSuccess) e = cudaEventSynchronize(ev[1]);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(ms_out, ev[0], ev[1]);
+  for (cudaEvent_t x : ev)
+    if (x) cudaEventDestroy(x);
+  if (e != cudaSuccess) return cuda_fail(e, "insert request-ceiling probe");
+  return GS_OK;
+  GS_GUARD_END
+}
+
+gs_status gs_query_request_ceiling(const gs_sketch* sk, int64_t d, void* window, size_t window_bytes, float* ms_out,
+                                   gs_stream stream) {
+  GS_GUARD_BEGIN
+  GS_TRY(check_sketch(sk));
+  GS_TRY(check_d(d));
+  if (!window || !aligned(window, 256)) return fail(GS_ERR_INVALID_ARG, "window is NULL or not 256-byte aligned");
+  if (window_bytes < 65536) return fail(GS_ERR_INVALID_ARG, "window too small: need 65536 bytes");
+  if (!ms_out) return fail(GS_ERR_INVALID_ARG, "ms_out is NULL");
+  if ((sk->c & (sk->c - 1)) != 0) return fail(GS_ERR_INVALID_ARG, "the probe serves c a power of two");
+  cudaStream_t s = as_stream(stream);
+  cudaEvent_t ev[2] = {nullptr, nullptr};
+  cudaError_t e = cudaEventCreate(&ev[0]);
+  if (e == cudaSuccess) e = cudaEventCreate(&ev[1]);
+  if (e == cudaSuccess) e = cudaEventRecord(ev[0], s);
+  if (e == cudaSuccess)
+    e = gs::launch_query_ceiling_probe(sk->merged, sk->h, sk->r, (uint32_t)sk->c, d, static_cast<float*>(window),
+                                       (int64_t)(window_bytes / sizeof(float)), s);
+  if (e == cudaSuccess) e = cudaEventRecord(ev[1], s);
+  if (e == cudaSuccess) e = cudaEventSynchronize(ev[1]);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(ms_out, ev[0], ev[1]);
+  for (cudaEvent_t x : ev)
+    if (x) cudaEventDestroy(x);
+  if (e != cudaSuccess) return cuda_fail(e, "query request-ceiling probe");
+  return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_hash_eval(const gs_sketch* sk, const int64_t* coords, int64_t n, int32_t* bucket_out, int8_t* sign_out,

@@ -82,6 +82,7 @@ struct InsertParams {
   int32_t j0, j1;    // rows inserted by this launch: [j0, j1)
   uint32_t c, cmask;
   float rho;
+  int64_t winmask;   // request-ceiling probe only: vector offsets are taken modulo winmask + 1
   HashCoeffs h;
 };
 
@@ -117,6 +118,15 @@ cudaError_t launch_accumulate(float* u, float* e, const float* g, int64_t d, flo
 // acc: accumulate (read g, u, e; write u, e) before inserting; otherwise insert e as it is.
 cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool acc, bool vec, cudaStream_t s);
 cudaError_t launch_insert_lane(const InsertParams& p, int W, cudaStream_t s);
+// The fused insert's instruction stream with every vector access at offset i & p.winmask (the
+// vectors are windows of winmask + 1 floats, 16-byte aligned): the same loads, stores and
+// cell reductions, with the streams held in L2.  W in {4, 8, 16}, c a power of two.
+cudaError_t launch_insert_ceiling_probe(const InsertParams& p, int W, bool acc, cudaStream_t s);
+// Shared-memory-staged insert of the (already accumulated) vectors p.e[0..nw) into rows
+// [j0, j1) of a W-wide group table; needs a tile of c * wt * 4 bytes (staged_tile_width).
+constexpr size_t kStagedSmemBytes = size_t(200) << 10;
+int staged_tile_width(uint32_t c, int W);   // workers per tile, 0 when no tile fits
+cudaError_t launch_insert_staged(const InsertParams& p, int W, cudaStream_t s);
 cudaError_t launch_hash_eval(const HashCoeffs& h, int r, uint32_t c, const int64_t* coords,
                              int64_t n, int32_t* bucket_out, int8_t* sign_out, cudaStream_t s);
 cudaError_t launch_merge(const MergeParams& p, int W, cudaStream_t s);
@@ -132,15 +142,21 @@ cudaError_t launch_query_at(const float* T, const HashCoeffs& h, int r, uint32_t
 cudaError_t launch_add_sparse(float* T, const HashCoeffs& h, int r, uint32_t c, const int64_t* idx, const float* vals,
                               int64_t k, float scale, cudaStream_t s);
 cudaError_t launch_take(const float* src, int64_t n, const int64_t* idx, int64_t k, float* out, cudaStream_t s);
+// marks (nullable): three events recorded, when set, before the query, between the query
+// (sample, median query, repair check) and the selection, and after the selection.
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, cudaStream_t s);
+                              void* workspace, cudaStream_t s, const cudaEvent_t* marks = nullptr);
+// Request-ceiling probe of the median query: its loads (all r rows) without median, store or
+// histogram; out receives one float per CTA (out_floats must cover the grid).  c a power of two.
+cudaError_t launch_query_ceiling_probe(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
+                                       float* out, int64_t out_floats, cudaStream_t s);
 // HEAVYMIX selection (Alg. 2 as printed) from the merged table; l2sq_out (device double,
 // nullable) receives the sketch's estimate of ||g||^2.
 size_t heavymix_workspace_bytes(int64_t d, int64_t k);
 cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
                                   int64_t k, uint64_t fill_seed, int64_t* idx_out, float* est_out, double* l2sq_out,
-                                  void* workspace, cudaStream_t s);
+                                  void* workspace, cudaStream_t s, const cudaEvent_t* marks = nullptr);
 
 // Same pipeline with its scratch in a fixed device array (no allocation); est_out required,
 // d <= GS_NOALLOC_MAX_DIM.  The first call on a device looks up the array's address.

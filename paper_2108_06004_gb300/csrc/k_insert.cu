@@ -55,26 +55,31 @@ __global__ void __launch_bounds__(kBlock) k_accumulate(float* __restrict__ u,
   }
 }
 
-// Load (and with ACC, update and store) four consecutive coordinates of lane w.
-template <bool ACC, bool VEC>
+// Load (and with ACC, update and store) four consecutive coordinates of lane w.  WIN (the
+// request-ceiling probe only) folds the vector offset into a window of prm.winmask + 1 floats.
+template <bool ACC, bool VEC, bool WIN = false>
 __device__ __forceinline__ void load_lane(const InsertParams& prm, int w, int64_t i0,
                                           int64_t d, float (&ev)[4]) {
   if (VEC && i0 + 4 <= d) {
-    float4 e4 = __ldcs(reinterpret_cast<const float4*>(prm.e[w] + i0));
+    const int64_t ia = WIN ? (i0 & prm.winmask) : i0;
+    float4 e4 = __ldcs(reinterpret_cast<const float4*>(prm.e[w] + ia));
     if (ACC) {
-      float4 g4 = __ldcs(reinterpret_cast<const float4*>(prm.g[w] + i0));
-      float4 u4 = __ldcs(reinterpret_cast<const float4*>(prm.u[w] + i0));
+      float4 g4 = __ldcs(reinterpret_cast<const float4*>(prm.g[w] + ia));
+      float4 u4 = __ldcs(reinterpret_cast<const float4*>(prm.u[w] + ia));
       acc1(prm.rho, u4.x, e4.x, g4.x);
       acc1(prm.rho, u4.y, e4.y, g4.y);
       acc1(prm.rho, u4.z, e4.z, g4.z);
       acc1(prm.rho, u4.w, e4.w, g4.w);
-      __stcs(reinterpret_cast<float4*>(prm.u[w] + i0), u4);
-      __stcs(reinterpret_cast<float4*>(prm.e[w] + i0), e4);
+      __stcs(reinterpret_cast<float4*>(prm.u[w] + ia), u4);
+      __stcs(reinterpret_cast<float4*>(prm.e[w] + ia), e4);
     }
     ev[0] = e4.x;
     ev[1] = e4.y;
     ev[2] = e4.z;
     ev[3] = e4.w;
+  } else if (WIN) {
+#pragma unroll
+    for (int t = 0; t < 4; ++t) ev[t] = 0.f;  // the probe's ragged tail carries no requests
   } else {
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
@@ -146,7 +151,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_const
 // at offset 4*sub of the cell, so the G lanes of the group cover the whole cell in the same
 // instruction.  The hash is evaluated by every lane of the group (issue slots are not the
 // bound here).
-template <int W, bool ACC, bool VEC, bool POW2>
+template <int W, bool ACC, bool VEC, bool POW2, bool WIN = false>
 __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_constant__ InsertParams prm) {
   grid_begin();
   constexpr int G = W / 4;
@@ -161,7 +166,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_
     for (int w4 = 0; w4 < 4; ++w4) {
       const int w = sub * 4 + w4;
       if (w < prm.nw) {
-        load_lane<ACC, VEC>(prm, w, i0, d, ev[w4]);
+        load_lane<ACC, VEC, WIN>(prm, w, i0, d, ev[w4]);
       } else {
 #pragma unroll
         for (int t = 0; t < 4; ++t) ev[w4][t] = 0.f;
@@ -219,6 +224,67 @@ __global__ void __launch_bounds__(kBlock) k_insert_lane(const __grid_constant__ 
         }
       }
     }
+  }
+}
+
+// Shared-memory-staged insert (the alternative to k_accumulate_insert_coop's direct cell
+// reductions; the error vectors are already accumulated).  blockIdx.y is the row j and
+// blockIdx.z a tile of WT adjacent workers of the group; blockIdx.x a contiguous chunk of the
+// coordinates.  The CTA keeps row j of its WT workers' tables in shared memory ([c][WT] fp32),
+// adds its chunk into it with shared-memory atomics, then flushes the tile into the group
+// table with one WT-wide vector reduction per bucket (buckets the chunk never touched are
+// skipped).  Only for tables whose tile fits: c * WT * 4 bytes of dynamic shared memory.
+template <int WT, bool POW2>
+__global__ void __launch_bounds__(kBlock) k_insert_staged(const __grid_constant__ InsertParams prm, int W,
+                                                         int64_t chunk) {
+  grid_begin();
+  extern __shared__ float tile[];
+  const int j = blockIdx.y;
+  const int w0 = blockIdx.z * WT;
+  const uint32_t c = prm.c;
+  for (uint32_t b = threadIdx.x; b < c * WT; b += blockDim.x) tile[b] = 0.f;
+  __syncthreads();
+  const int64_t d = prm.d;
+  const int64_t a0 = (int64_t)blockIdx.x * chunk;
+  const int64_t a1 = a0 + chunk < d ? a0 + chunk : d;
+  const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
+  for (int64_t i0 = a0 + 4 * (int64_t)threadIdx.x; i0 < a1; i0 += 4 * (int64_t)blockDim.x) {
+    const int tmax = (a1 - i0 < 4) ? (int)(a1 - i0) : 4;
+    float ev[WT][4];
+#pragma unroll
+    for (int w = 0; w < WT; ++w) {
+#pragma unroll
+      for (int t = 0; t < 4; ++t) ev[w][t] = (w0 + w < prm.nw && t < tmax) ? prm.e[w0 + w][i0 + t] : 0.f;
+    }
+    uint64_t x = affine61(a, prm.h.b[j], (uint32_t)i0);
+    uint64_t y = affine61(a2, prm.h.b2[j], (uint32_t)i0);
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      if (t < tmax) {
+        const uint32_t bk = bucket_of<POW2>(x, c, prm.cmask);
+        const uint32_t sb = signbit_of(y);
+#pragma unroll
+        for (int w = 0; w < WT; ++w) atomicAdd(&tile[bk * WT + w], apply_sign(ev[w][t], sb));
+        x = step61(x, a);
+        y = step61(y, a2);
+      }
+    }
+  }
+  __syncthreads();
+  float* row = prm.table + (size_t)j * c * W + w0;
+  for (uint32_t b = threadIdx.x; b < c; b += blockDim.x) {
+    float v[WT];
+    bool any = false;
+#pragma unroll
+    for (int w = 0; w < WT; ++w) {
+      v[w] = tile[b * WT + w];
+      any = any || v[w] != 0.f;
+    }
+    if (!any) continue;
+    float* cell = row + (size_t)b * W;
+    if (WT == 4) red_add_v4(cell, v[0], v[WT > 1 ? 1 : 0], v[WT > 2 ? 2 : 0], v[WT > 3 ? 3 : 0]);
+    else if (WT == 2) red_add_v2(cell, v[0], v[WT > 1 ? 1 : 0]);
+    else red_add_f32(cell, v[0]);
   }
 }
 
@@ -295,6 +361,77 @@ cudaError_t launch_accumulate_insert(const InsertParams& p, int W, bool acc, boo
     case 4: return launch_ai_acc<4>(p, acc, vec, s);
     case 8: return launch_ai_acc<8>(p, acc, vec, s);
     case 16: return launch_ai_acc<16>(p, acc, vec, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int W>
+cudaError_t launch_ceiling_w(const InsertParams& p, bool acc, cudaStream_t s) {
+  auto kern = acc ? k_accumulate_insert_coop<W, true, true, true, true> : k_accumulate_insert_coop<W, false, true, true, true>;
+  // the same grid as the insert it stands for
+  auto real = acc ? k_accumulate_insert_coop<W, true, true, true> : k_accumulate_insert_coop<W, false, true, true>;
+  const int grid = grid_for(real, (p.d + 3) / 4 * (W / 4), kBlock);
+  launch(kern, grid, kBlock, s, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_insert_ceiling_probe(const InsertParams& p, int W, bool acc, cudaStream_t s) {
+  if (!is_pow2(p.c)) return cudaErrorInvalidValue;
+  switch (W) {
+    case 4: return launch_ceiling_w<4>(p, acc, s);
+    case 8: return launch_ceiling_w<8>(p, acc, s);
+    case 16: return launch_ceiling_w<16>(p, acc, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+int staged_tile_width(uint32_t c, int W) {
+  int wt = W < 4 ? W : 4;
+  while (wt > 1 && (size_t)c * wt * sizeof(float) > kStagedSmemBytes) wt /= 2;
+  return (size_t)c * wt * sizeof(float) <= kStagedSmemBytes ? wt : 0;
+}
+
+template <int WT, bool POW2>
+cudaError_t launch_staged_t(const InsertParams& p, int W, cudaStream_t s) {
+  auto kern = k_insert_staged<WT, POW2>;
+  const size_t smem = (size_t)p.c * WT * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  // about two CTAs per SM over all (row, worker tile) pairs, at least one chunk
+  const int tiles = (p.j1 - p.j0) * (W / WT);
+  int64_t nchunk = (2 * (int64_t)device_info().sms + tiles - 1) / tiles;
+  int64_t chunk = (p.d + nchunk - 1) / nchunk;
+  chunk = (chunk + 3) / 4 * 4;
+  nchunk = (p.d + chunk - 1) / chunk;
+  InsertParams q = p;
+  q.table = p.table + (size_t)p.j0 * p.c * W;  // blockIdx.y counts rows from j0
+  for (int j = p.j0; j < p.j1; ++j) {  // coefficients re-based so that row blockIdx.y is row j
+    q.h.a[j - p.j0] = p.h.a[j];
+    q.h.b[j - p.j0] = p.h.b[j];
+    q.h.a2[j - p.j0] = p.h.a2[j];
+    q.h.b2[j - p.j0] = p.h.b2[j];
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)nchunk, (unsigned)(p.j1 - p.j0), (unsigned)(W / WT));
+  cfg.blockDim = dim3(kBlock);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, q, W, chunk);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t launch_insert_staged(const InsertParams& p, int W, cudaStream_t s) {
+  const int wt = staged_tile_width(p.c, W);
+  const bool pow2 = is_pow2(p.c);
+  switch (wt) {
+    case 4: return pow2 ? launch_staged_t<4, true>(p, W, s) : launch_staged_t<4, false>(p, W, s);
+    case 2: return pow2 ? launch_staged_t<2, true>(p, W, s) : launch_staged_t<2, false>(p, W, s);
+    case 1: return pow2 ? launch_staged_t<1, true>(p, W, s) : launch_staged_t<1, false>(p, W, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -412,6 +412,44 @@ __global__ void __launch_bounds__(kBlock) k_qsample(const __grid_constant__ Quer
   }
 }
 
+// Request-ceiling probe of the query (measurement aid): the loads of k_query with every row
+// read (the same grid, hash buckets and incremental form), without the median, the estimate
+// store or the histogram.  Each CTA writes the sum of what it read to out[blockIdx.x], so that
+// the loads cannot be dropped.
+template <int R>
+__global__ void __launch_bounds__(kBlock) k_gather_probe(const __grid_constant__ QueryParams prm, float* out) {
+  grid_begin();
+  __shared__ float warp_sum[kBlock / 32];
+  const int64_t d = prm.d, nq = (d + 3) / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  float acc = 0.f;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nq; q += stride) {
+    const int64_t i0 = q * 4;
+    const int tmax = d - i0 < 4 ? (int)(d - i0) : 4;
+#pragma unroll
+    for (int j = 0; j < R; ++j) {
+      uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+      const float* row = prm.T + (size_t)j * prm.c;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        if (t < tmax) {
+          acc += __ldg(row + ((uint32_t)x & prm.cmask));
+          x = step61(x, prm.h.a[j]);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(kFull, acc, o);
+  if ((threadIdx.x & 31) == 0) warp_sum[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+    for (int w = 0; w < kBlock / 32; ++w) t += warp_sum[w];
+    out[blockIdx.x] = t;
+  }
+}
+
 // General path: any r <= 16 and any c (bucket by 64-bit remainder).
 __global__ void __launch_bounds__(kBlock) k_query_generic(const __grid_constant__ QueryParams prm) {
   grid_begin();
@@ -1032,6 +1070,24 @@ uint32_t sample_rank(int64_t d, int64_t k) {
   return j <= (double)n_s ? (uint32_t)j : 0u;
 }
 
+template <int R>
+cudaError_t launch_gather_probe_r(const QueryParams& p, float* out, int64_t out_floats, cudaStream_t s) {
+  auto kern = k_gather_probe<R>;
+  const int grid = persistent_grid(k_query<R>, (p.d + 3) / 4, kBlock);  // the query's grid
+  if (grid > out_floats) return cudaErrorInvalidValue;
+  launch(kern, grid, kBlock, s, p, out);
+  return cudaGetLastError();
+}
+
+typedef cudaError_t (*ProbeLauncher)(const QueryParams&, float*, int64_t, cudaStream_t);
+
+template <int... Rs>
+struct ProbeTable {
+  static constexpr ProbeLauncher table[sizeof...(Rs)] = {&launch_gather_probe_r<Rs>...};
+};
+template <int... Rs>
+constexpr ProbeLauncher ProbeTable<Rs...>::table[sizeof...(Rs)];
+
 // Pruning applies on the fast path (c a power of two) with at least three rows, and from
 // 2^22 coordinates up: below that the query takes a few tens of microseconds and the repair
 // kernel's launch costs more than the skipped rows save (measured on the 2^20 workload).
@@ -1110,6 +1166,11 @@ size_t query_topk_workspace_bytes(int64_t d, int64_t k) {
 
 namespace {
 
+// Records marks[i] on s when the caller passed marks and set that entry (while a plan is captured).
+cudaError_t mark(const cudaEvent_t* marks, int i, cudaStream_t s) {
+  return (marks && marks[i]) ? cudaEventRecordWithFlags(marks[i], s, cudaEventRecordExternal) : cudaSuccess;
+}
+
 // Histograms, state and both bitmaps back to zero.
 cudaError_t clear_selection(const Workspace& w, cudaStream_t s) {
   cudaError_t err = cudaMemsetAsync(w.hist, 0, 5 * kBins * sizeof(uint32_t), s);
@@ -1143,11 +1204,12 @@ cudaError_t select_from_keys(const Workspace& w, const float* src, int vec, uint
 
 cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, uint32_t c,
                               int64_t d, int64_t k, int64_t* idx_out, float* est_out,
-                              void* workspace, cudaStream_t s) {
+                              void* workspace, cudaStream_t s, const cudaEvent_t* marks) {
   Workspace w = carve(workspace, d);
   float* est = est_out ? est_out : w.est;
   cudaError_t err = clear_selection(w, s);
   if (err != cudaSuccess) return err;
+  if ((err = mark(marks, 0, s)) != cudaSuccess) return err;
 
   QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
   // rows are pruned only while the estimate stays internal: a caller's est_out gets every value
@@ -1162,7 +1224,17 @@ cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, u
     using T = RepairTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
     if ((err = T::table[r - 1](qp, w.hist + 3 * kBins, s)) != cudaSuccess) return err;
   }
-  return select_from_keys(w, est, qp.vec, 0x7FFFFFFFu, d, k, idx_out, s);
+  if ((err = mark(marks, 1, s)) != cudaSuccess) return err;
+  if ((err = select_from_keys(w, est, qp.vec, 0x7FFFFFFFu, d, k, idx_out, s)) != cudaSuccess) return err;
+  return mark(marks, 2, s);
+}
+
+cudaError_t launch_query_ceiling_probe(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
+                                       float* out, int64_t out_floats, cudaStream_t s) {
+  if (!is_pow2(c) || r < 1 || r > GS_MAX_ROWS) return cudaErrorInvalidValue;
+  const QueryParams qp = make_query_params(merged, h, r, c, d, 1, nullptr, nullptr, nullptr);
+  using T = ProbeTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
+  return T::table[r - 1](qp, out, out_floats, s);
 }
 
 size_t heavymix_workspace_bytes(int64_t d, int64_t k) {
@@ -1171,7 +1243,7 @@ size_t heavymix_workspace_bytes(int64_t d, int64_t k) {
 
 cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int r, uint32_t c, int64_t d,
                                   int64_t k, uint64_t fill_seed, int64_t* idx_out, float* est_out, double* l2sq_out,
-                                  void* workspace, cudaStream_t s) {
+                                  void* workspace, cudaStream_t s, const cudaEvent_t* marks) {
   Workspace w = carve(workspace, d);
   char* extra = static_cast<char*>(workspace) + query_topk_workspace_bytes(d, k);
   uint32_t* keys = reinterpret_cast<uint32_t*>(extra);
@@ -1180,6 +1252,7 @@ cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int 
   float* est = est_out ? est_out : w.est;
   cudaError_t err = clear_selection(w, s);
   if (err == cudaSuccess) err = cudaMemsetAsync(sumsq, 0, 256, s);
+  if (err == cudaSuccess) err = mark(marks, 0, s);
   if (err != cudaSuccess) return err;
 
   // the threshold first (it reads only the table), so that the query can skip rows below it
@@ -1194,7 +1267,11 @@ cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int 
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
   launch(k_heavy_keys, persistent_grid(k_heavy_keys, d, kBlock), kBlock, s, est, d, theta, fill_seed, keys, w.hist,
                                                                            w.st, (uint32_t)k);
-  return select_from_keys(w, reinterpret_cast<const float*>(keys), 1, 0xFFFFFFFFu, d, k, idx_out, s);
+  if ((err = mark(marks, 1, s)) != cudaSuccess) return err;
+  if ((err = select_from_keys(w, reinterpret_cast<const float*>(keys), 1, 0xFFFFFFFFu, d, k, idx_out, s)) !=
+      cudaSuccess)
+    return err;
+  return mark(marks, 2, s);
 }
 
 // ---- scratch without allocation ---------------------------------------------------------

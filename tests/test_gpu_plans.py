@@ -309,3 +309,84 @@ def test_step_plan_repairs_a_prune_key_above_the_threshold(gs, H):
     finally:
         gs.gs_plan_destroy(plan)
         run.close()
+
+
+def test_step_plan_query_times(gs, H):
+    """GS_PLAN_TIME_QUERY: one positive median-query and selection duration per launch; a plan
+    created without the flag rejects the request."""
+    run = H.new_run(2, 8192, 3, 512, 16, 4)
+    g = [torch.randn(8192, device="cuda") for _ in range(2)]
+    flags = gs.GS_PLAN_TIME_INSERT | gs.GS_PLAN_TIME_QUERY
+    plan = gs.gs_step_plan_create(run.sketch, run.us, run.es, g, 8192, 0.9, 16, run.idx, run.vals, None, None, 0.0,
+                                  run.ws, flags=flags)
+    plain = gs.gs_step_plan_create(run.sketch, run.us, run.es, g, 8192, 0.9, 16, run.idx, run.vals, None, None, 0.0,
+                                   run.ws, flags=gs.GS_PLAN_TIME_INSERT)
+    try:
+        for _ in range(5):
+            gs.gs_plan_launch(plan)
+        q, s = gs.gs_plan_query_times(plan, 10)
+        assert len(q) == len(s) == 5 and all(x > 0 for x in q + s)
+        assert len(gs.gs_plan_insert_times(plan, 10)) == 5
+        gs.gs_plan_launch(plain)
+        with pytest.raises(gs.GsError):
+            gs.gs_plan_query_times(plain, 4)
+    finally:
+        gs.gs_plan_destroy(plan)
+        gs.gs_plan_destroy(plain)
+        run.close()
+
+
+def test_heavymix_step_and_plan(gs, H):
+    """A step with the HEAVYMIX selection, first through gs_heavymix_step and then twice through
+    its plan (gradients refilled in place), each against the fp64 oracle: momentum and error
+    bit-exact off the selection and zero on it, the estimate (kept in the workspace) within its
+    band, the selection exactly the rule applied to the GPU's own estimate and l2sq, and equal
+    to the oracle's wherever H agrees (band coordinates are the only free choices)."""
+    from tests.test_gpu_parity import _check_heavymix_against_oracle
+    w = workloads.get_config("tiny-2^20")
+    P, d, r, c, k, seed, fill_seed = 4, 300_007, 5, 4096, 300, 51, 2**40 + 7
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, k, seed, rho=w.rho)
+    ws = torch.empty(gs.gs_heavymix_step_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+    l2 = torch.empty(1, dtype=torch.float64, device="cuda")
+    gbuf = [torch.empty(d, dtype=torch.float32, device="cuda") for _ in range(P)]
+    plan = gs.gs_heavymix_step_plan_create(run.sketch, run.us, run.es, gbuf, d, w.rho, k, fill_seed, run.idx,
+                                           run.vals, l2, ws, flags=gs.GS_PLAN_TIME_INSERT | gs.GS_PLAN_TIME_QUERY)
+    try:
+        hashes = oracle.hash_rows(coeffs, c, np.arange(d, dtype=np.uint64))
+        for t in range(3):
+            grads = workloads.make_gradients(w, t, range(P), d=d)
+            for b, g in zip(gbuf, grads):
+                b.copy_(torch.from_numpy(g))
+            us0 = [H.host(u) for u in run.us]
+            es0 = [H.host(e) for e in run.es]
+            if t == 0:
+                gs.gs_heavymix_step(run.sketch, run.us, run.es, gbuf, d, w.rho, k, fill_seed, run.idx, run.vals, l2, ws)
+            else:
+                gs.gs_plan_launch(plan)
+            torch.cuda.synchronize()
+            idx, vals, l2sq = H.host(run.idx), H.host(run.vals), float(l2.item())
+            est = H.host(ws[: 4 * d].view(torch.float32)).copy()      # d < 2^22: every row read
+            assert np.array_equal(idx, oracle.heavymix_select(est, l2sq, k, fill_seed))
+            pre = [oracle.accumulate(u0, e0, g, w.rho) for u0, e0, g in zip(us0, es0, grads)]
+            tabs = [oracle.sketch(e1, coeffs, c, hashes) for _, e1 in pre]
+            T = oracle.merge_tree([a for a, _ in tabs])
+            A = oracle.merge_tree([b for _, b in tabs])
+            idx_o, est_o, l2_o = oracle.heavymix(T, coeffs, d, k, fill_seed, hashes)
+            band = oracle.cell_band(A, coeffs, np.arange(d))
+            assert np.all(np.abs(est.astype(np.float64) - est_o) <= band)
+            assert abs(l2sq - l2_o) <= 1e-4 * l2_o
+            _check_heavymix_against_oracle(H, idx, est, l2sq, est_o, l2_o, band, k, fill_seed)
+            sel = np.zeros(d, bool)
+            sel[idx] = True
+            for p, (u1, e1) in enumerate(pre):
+                gu, ge = H.host(run.us[p]), H.host(run.es[p])
+                assert np.array_equal(gu[~sel].view(np.uint32), u1[~sel].view(np.uint32))
+                assert np.array_equal(ge[~sel].view(np.uint32), e1[~sel].view(np.uint32))
+                assert np.all(gu[sel] == 0) and np.all(ge[sel] == 0)
+            H.check_vals(vals, idx, [e1 for _, e1 in pre])
+        q, s = gs.gs_plan_query_times(plan, 10)
+        assert len(q) == 2 and all(x > 0 for x in q + s)
+    finally:
+        gs.gs_plan_destroy(plan)
+        run.close()

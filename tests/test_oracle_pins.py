@@ -514,3 +514,41 @@ def test_sketched_state_removal_and_momentum_closed_form():
         assert np.all(oracle.query_at(U, co, rest) == (2 - 2.0 ** (1 - t)) / 4)
         assert np.all(oracle.query_at(E, co, rest) == (2 * t - 2 + 2.0 ** (1 - t)) / 4)
         assert oracle.query_at(E, co, [t - 1])[0] == 0 and oracle.query_at(U, co, [t - 1])[0] == 0
+
+
+# ---- pieces of a long vector (linearity over disjoint coordinate ranges) ------------------
+
+def test_sketch_in_pieces_equals_whole():
+    """Sec. III-A's linearity over a partition of the coordinates: sketching x piece by piece,
+    each piece hashed at its own global coordinates, and summing gives exactly the sketch of x
+    (dyadic values: every sum is exact in fp64).  The same holds for the magnitude table, and
+    the median query evaluated piece by piece concatenates to the whole query."""
+    rng = np.random.default_rng(31)
+    d, r, c = 10_007, 5, 97
+    co = oracle.derive_coefficients(r, 31)
+    x = _dyadic(rng, d, -1000, 1000, 2.0**-10)
+    T, A = oracle.sketch(x, co, c)
+    Tp, Ap = np.zeros_like(T), np.zeros_like(A)
+    cuts = [0, 1, 17, 4096, 4097, 9000, d]
+    for a, b in zip(cuts[:-1], cuts[1:]):
+        t, m = oracle.sketch(x[a:b], co, c, idx=np.arange(a, b))
+        Tp += t
+        Ap += m
+    assert np.array_equal(T, Tp) and np.array_equal(A, Ap)
+    est = oracle.query(T, co, d)
+    parts = [oracle.query(T, co, b - a, idx=np.arange(a, b)) for a, b in zip(cuts[:-1], cuts[1:])]
+    assert np.array_equal(est, np.concatenate(parts))
+    # a piece hashed at the wrong coordinates (its local 0 .. n-1) does not give the sketch
+    bad = sum(oracle.sketch(x[a:b], co, c)[0] for a, b in zip(cuts[:-1], cuts[1:]))
+    assert not np.array_equal(bad, T)
+
+
+def test_topk_by_threshold_equals_topk():
+    """The partition-based top-k returns exactly the sorted definition's set, with heavy ties
+    (including ties at the k-th value) and with k = 1 and k = d."""
+    rng = np.random.default_rng(32)
+    for trial in range(40):
+        d = int(rng.integers(1, 400))
+        est = rng.integers(-6, 7, d).astype(np.float64) * (0.5 if trial % 2 else 1.0)
+        for k in {1, d, int(rng.integers(1, d + 1))}:
+            assert np.array_equal(oracle.topk_by_threshold(est, k), oracle.topk(est, k))
