@@ -67,6 +67,11 @@ def parse_args(argv=None):
                     help="which form of the step to time (the default is the headline path)")
     ap.add_argument("--eager", action="store_true",
                     help="one library call per kernel instead of a captured plan per step")
+    ap.add_argument("--group-width", type=int, default=0,
+                    help="workers interleaved per sketch table (0: the library's choice)")
+    ap.add_argument("--insert", default="direct", choices=["direct", "staged"],
+                    help="staged: the shared-memory-staged insert (gs_accumulate_insert_staged; eager, and only "
+                         "where a table row fits a shared-memory tile)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-per-config", action="store_true", help="time only the headline workload")
@@ -237,9 +242,13 @@ class Runner:
     batch's fresh gradients are drawn on the device into one shared buffer set (timed with
     their own events, outside the insert's) and then inserted; such steps run eagerly."""
 
-    def __init__(self, gs, w, variant, eager, rank, dev, stream, steps_needed, want_host_pool):
+    def __init__(self, gs, w, variant, eager, rank, dev, stream, steps_needed, want_host_pool, staged=False,
+                 group_width=0):
         import torch
         self.gs, self.w, self.variant, self.dev, self.stream = gs, w, variant, dev, stream
+        self.staged = staged
+        if staged:
+            eager = True
         self.rank = rank
         P, d, r, c, k = w.P, w.d, w.r, w.c, w.k
         self.streamed = bool(w.worker_batch) and w.worker_batch < P
@@ -267,11 +276,12 @@ class Runner:
         self.us = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
         self.es = [torch.zeros(d, dtype=torch.float32, device=dev) for _ in range(P)]
         gs = self.gs
-        self.sk = gs.gs_sketch_create(r, c, 20210813, P, 0)
+        self.sk = gs.gs_sketch_create(r, c, 20210813, P, group_width)
         info = gs.gs_sketch_info(self.sk)
         self.W, self.rpp = info["group_width"], info["rows_per_pass"]
         self.groups = (P + self.W - 1) // self.W
-        self.passes = -(-r // self.rpp)
+        ip = gs.gs_sketch_insert_passes(self.sk)
+        self.passes, self.bucket_parts = ip["passes"], ip["bucket_parts"]
         ws_bytes = gs.gs_step_workspace_size(d, k)
         if variant == "heavymix":
             ws_bytes = max(ws_bytes, gs.gs_query_heavymix_workspace_size(d, k))
@@ -341,7 +351,8 @@ class Runner:
             ins = _event_pair(record)
             if ins:
                 ins[0].record(s)
-            gs.gs_accumulate_insert(self.sk, 0, self.us, self.es, self.dev_pool[t % self.nsteps_pool], d, rho, s)
+            insert = gs.gs_accumulate_insert_staged if self.staged else gs.gs_accumulate_insert
+            insert(self.sk, 0, self.us, self.es, self.dev_pool[t % self.nsteps_pool], d, rho, s)
             if ins:
                 ins[1].record(s)
                 self.ev["insert"].append([ins])
@@ -465,17 +476,20 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
     w = run.w
     P, d, r = w.P, w.d, w.r
     per_wc = 4.0 if variant == "sketched_state" else 20.0
-    moved_wc = per_wc + 4.0 * (run.passes - 1)
+    moved_wc = per_wc + 4.0 * (run.passes - 1)   # every pass after the first re-reads e (or g)
     phase_s = ph["insert"] / 1e3
     phase_bytes = per_wc * P * d
     k1_gbs = phase_bytes / phase_s / 1e9
     cells = d * r * run.groups
-    nl = run.groups * run.passes * (w.P // run.batch if run.streamed else 1)
+    nl = run.groups * run.passes
     k1 = {
-        "kernel": ("k_accumulate_insert_coop (insert only" if variant == "sketched_state" else
+        "kernel": ("k_accumulate + k_insert_staged (S1, then S2 staged in shared memory" if run.staged else
+                   "k_accumulate_insert_coop (insert only" if variant == "sketched_state" else
                    "k_accumulate_insert_coop (fused S1+S2") + f", W={run.W}), the insert phase of a step: "
-                  f"{run.groups} group(s) x {run.passes} row pass(es)",
-        "row_passes": run.passes, "groups": run.groups, "launches_per_phase": nl,
+                  f"{run.groups} group(s) x {run.passes} pass(es)" +
+                  (f" (rows in {run.bucket_parts} bucket ranges)" if run.bucket_parts > 1 else ""),
+        "row_passes": run.passes, "bucket_parts_per_row": run.bucket_parts, "groups": run.groups,
+        "launches_per_phase": nl,
         "algorithmic_bytes_per_worker_coord": per_wc, "moved_bytes_per_worker_coord": moved_wc,
         "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
         "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,
@@ -548,11 +562,11 @@ def probe_ceilings(run: Runner, reps: int = 3) -> dict:
 
 
 def measure(gs, w, variant, eager, steps, warmup, world, rank, dev, stream, peaks, peak_kind, sampler=None,
-            want_e2e=False, probes=True):
+            want_e2e=False, probes=True, staged=False, group_width=0):
     """Time one workload; returns (summary dict, Runner still open for e2e)."""
     import torch
     want_host = want_e2e and variant == "error_feedback"
-    run = Runner(gs, w, variant, eager, rank, dev, stream, steps + warmup, want_host)
+    run = Runner(gs, w, variant, eager, rank, dev, stream, steps + warmup, want_host, staged, group_width)
     flush = None
     streamed_bytes = w.P * w.d * 12
     if streamed_bytes < 2 * L2_BYTES:
@@ -685,12 +699,16 @@ def run_ours(args):
     sampler = None if quick else ClockSampler(gpu_uuid(dev))
     if sampler:
         sampler.start()
+    staged = args.insert == "staged"
+    if staged and (variant != "error_feedback" or (w.worker_batch and w.worker_batch < w.P)):
+        raise SystemExit("--insert staged applies to the error_feedback step of a workload with all workers resident")
     res, run = measure(gs, w, variant, args.eager, args.steps, args.warmup, world, rank, dev, stream, peaks,
-                       peak_kind, sampler, want_e2e=not (args.no_e2e or quick), probes=not quick)
+                       peak_kind, sampler, want_e2e=not (args.no_e2e or quick) and not staged,
+                       probes=not quick, staged=staged, group_width=args.group_width)
     clocks = sampler.stop() if sampler else None
 
     e2e = None
-    if not args.no_e2e and not quick and variant == "error_feedback" and not run.streamed:
+    if not args.no_e2e and not quick and variant == "error_feedback" and not run.streamed and not staged:
         e2e = e2e_measure(gs, run, args.steps, args.warmup, world, dev)
     W, groups = run.W, run.groups
     run.close()
@@ -698,7 +716,7 @@ def run_ours(args):
     torch.cuda.empty_cache()
 
     per_config = None
-    if not args.no_per_config and not quick and variant == "error_feedback":
+    if not args.no_per_config and not quick and variant == "error_feedback" and not staged:
         per_config = {}
         for name in sorted(workloads.CONFIGS, key=lambda n: workloads.CONFIGS[n].d):
             wc = workloads.get_config(name)
@@ -721,7 +739,7 @@ def run_ours(args):
         "metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": w.name, "variant": variant, "launch": res["launch"],
+        "config": {"workload": w.name, "variant": variant, "launch": res["launch"], "insert": args.insert,
                    "warmup_steps_run": res["warmup_steps_run"], "d": w.d, "P": w.P, "r": w.r, "c": w.c, "k": w.k,
                    "rho": w.rho, "group_width": W, "groups": groups,
                    "parallelism": f"replicas{world}" if world > 1 else "single-gpu",

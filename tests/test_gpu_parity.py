@@ -160,6 +160,50 @@ def test_accumulate_insert_merge(gs, H, P, W, d, r, c, passes):
         run.close()
 
 
+@pytest.mark.parametrize("P,W,d,r,c", [(4, 0, 1 << 20, 5, 1 << 14), (3, 4, 123_457, 5, 1000), (8, 8, 200_003, 3, 4096),
+                                       (16, 16, 90_001, 5, 1 << 12), (2, 1, 70_001, 4, 50_000), (9, 0, 65_537, 7, 3001)])
+def test_accumulate_insert_staged(gs, H, P, W, d, r, c):
+    """The shared-memory-staged insert: momentum and error bit-exact against the oracle's
+    accumulate, every worker-table cell within 1e-5 of its magnitude of the oracle's sketch, and
+    the same rejection as documented where a row does not fit a shared-memory tile."""
+    seed = P * 100 + r
+    rng = np.random.default_rng(seed)
+    coeffs = oracle.derive_coefficients(r, seed)
+    run = H.new_run(P, d, r, c, 1, seed, rho=0.9, group_width=W)
+    try:
+        W = gs.gs_sketch_info(run.sketch)["group_width"]
+        us = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        es = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        gr = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        for p in range(P):
+            run.us[p].copy_(torch.from_numpy(us[p]))
+            run.es[p].copy_(torch.from_numpy(es[p]))
+        gdev = [_dev(g) for g in gr]
+        split = W if P > W else P
+        gs.gs_accumulate_insert_staged(run.sketch, 0, run.us[:split], run.es[:split], gdev[:split], d, 0.9)
+        if split < P:
+            gs.gs_accumulate_insert_staged(run.sketch, split, run.us[split:], run.es[split:], gdev[split:], d, 0.9)
+        tabs = H.worker_tables(run, P, r, c)
+        for p in range(P):
+            u1, e1 = oracle.accumulate(us[p], es[p], gr[p], 0.9)
+            assert np.array_equal(H.host(run.us[p]).view(np.uint32), u1.view(np.uint32))
+            assert np.array_equal(H.host(run.es[p]).view(np.uint32), e1.view(np.uint32))
+            T, A = oracle.sketch(e1, coeffs, c)
+            H.check_cells(tabs[p], T, A, f"worker {p}")
+    finally:
+        run.close()
+
+
+def test_accumulate_insert_staged_rejects_large_rows(gs, H):
+    run = H.new_run(2, 4096, 3, 1 << 16, 1, 3)
+    try:
+        with pytest.raises(gs.GsError) as ei:
+            gs.gs_accumulate_insert_staged(run.sketch, 0, run.us, run.es, run.es, 4096, 0.9)
+        assert ei.value.status == gs.GS_ERR_INVALID_ARG
+    finally:
+        run.close()
+
+
 def test_accumulate_insert_unaligned(gs, H):
     """Vectors that start 4 bytes past a 16-byte boundary take the scalar load path of the
     fused kernel; the state stays bit-exact and the tables agree with the oracle."""

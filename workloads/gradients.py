@@ -95,6 +95,20 @@ def torch_seed(w: Workload, step: int, worker: int) -> int:
     return int(ss.generate_state(1, dtype=np.uint64)[0] & np.uint64((1 << 63) - 1))
 
 
+_DEVICE_SCALES: dict = {}
+
+
+def _device_scales(w: Workload, device):
+    """The per-coordinate block scales of ``w`` as an fp32 device vector (one per workload and
+    device, kept between calls)."""
+    import torch
+    key = (w.name, w.d, w.cid, str(device))
+    if key not in _DEVICE_SCALES:
+        _DEVICE_SCALES.clear()
+        _DEVICE_SCALES[key] = torch.from_numpy(_scale_vector(w)).to(device)
+    return _DEVICE_SCALES[key]
+
+
 def make_gradient_torch(w: Workload, step: int, worker: int, out):
     """Fill the fp32 device tensor ``out`` (length d) with a gradient of the same recipe as
     ``make_gradient``, drawn on the device by PyTorch's generator (a different stream of
@@ -108,12 +122,9 @@ def make_gradient_torch(w: Workload, step: int, worker: int, out):
     else:
         out.exponential_(1.0, generator=gen)
         flip = torch.empty_like(out).uniform_(0.0, 1.0, generator=gen) < 0.5
-        out[flip] = -out[flip]
+        torch.where(flip, -out, out, out=out)
         del flip
-    off = 0
-    for size, s in zip(w.blocks, block_scales(w).astype(np.float32)):
-        out[off:off + size].mul_(float(s))
-        off += size
+    out.mul_(_device_scales(w, out.device))
     pos, sgn = spike_positions(w)
     if pos.size:
         pt = torch.from_numpy(pos).to(out.device)
