@@ -280,8 +280,7 @@ class Runner:
         info = gs.gs_sketch_info(self.sk)
         self.W, self.rpp = info["group_width"], info["rows_per_pass"]
         self.groups = (P + self.W - 1) // self.W
-        ip = gs.gs_sketch_insert_passes(self.sk)
-        self.passes, self.bucket_parts = ip["passes"], ip["bucket_parts"]
+        self.passes = -(-r // self.rpp)
         ws_bytes = gs.gs_step_workspace_size(d, k)
         if variant == "heavymix":
             ws_bytes = max(ws_bytes, gs.gs_query_heavymix_workspace_size(d, k))
@@ -486,10 +485,8 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
         "kernel": ("k_accumulate + k_insert_staged (S1, then S2 staged in shared memory" if run.staged else
                    "k_accumulate_insert_coop (insert only" if variant == "sketched_state" else
                    "k_accumulate_insert_coop (fused S1+S2") + f", W={run.W}), the insert phase of a step: "
-                  f"{run.groups} group(s) x {run.passes} pass(es)" +
-                  (f" (rows in {run.bucket_parts} bucket ranges)" if run.bucket_parts > 1 else ""),
-        "row_passes": run.passes, "bucket_parts_per_row": run.bucket_parts, "groups": run.groups,
-        "launches_per_phase": nl,
+                  f"{run.groups} group(s) x {run.passes} row pass(es)",
+        "row_passes": run.passes, "groups": run.groups, "launches_per_phase": nl,
         "algorithmic_bytes_per_worker_coord": per_wc, "moved_bytes_per_worker_coord": moved_wc,
         "bound": "hbm", "achieved": round(k1_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
         "frac": round(k1_gbs / peaks["hbm_gbs"], 4), "peak_source": peak_kind,

@@ -71,8 +71,7 @@ typedef struct gs_plan gs_plan;     /* opaque: one step captured into a CUDA gra
  * together write a whole cell in one instruction); group_width 0 lets the library choose
  * (up to 16, no wider than the worker count rounded up to a power of two; 16 only when the
  * whole group table fits 48 MiB of L2, and halved while one table row exceeds 64 MiB).  The
- * fused insert updates as many rows per pass as fit 48 MiB, and at least one; a row larger
- * than 48 MiB is updated in bucket ranges, one per pass (gs_sketch_insert_passes).
+ * fused insert updates as many rows per pass as fit 48 MiB, and at least one.
  * On success *out owns device memory released by gs_sketch_destroy.
  * Errors: GS_ERR_INVALID_ARG (sizes, group_width not in {0,1,2,4,8,16}, out NULL),
  *         GS_ERR_OOM (allocation failed), GS_ERR_CUDA.  Synchronous. */
@@ -86,12 +85,6 @@ gs_status gs_sketch_destroy(gs_sketch* sketch);
  * fused insert updates per pass over the vectors. */
 gs_status gs_sketch_info(const gs_sketch* sketch, int32_t* r, int32_t* c, int32_t* workers,
                          int32_t* group_width, int32_t* rows_per_pass);
-
-/* Passes of the fused insert over one group's vectors: *passes slices of the table per insert
- * (the first accumulates, the later ones re-read the error vectors), and *bucket_parts, the
- * number of bucket ranges each row is split into when one row exceeds the 48 MiB pass budget
- * (1 otherwise).  Either pointer may be NULL. */
-gs_status gs_sketch_insert_passes(const gs_sketch* sketch, int32_t* passes, int32_t* bucket_parts);
 
 /* Host copy of the hash coefficients: out4r[4*j + {0,1,2,3}] = a_j, b_j, a'_j, b'_j
  * (host array of 4*r uint64).  Synchronous, no device work. */

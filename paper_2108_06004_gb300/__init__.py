@@ -40,7 +40,6 @@ SIGNATURES = {
     "gs_sketch_info": [_vp, ctypes.POINTER(_i32), ctypes.POINTER(_i32), ctypes.POINTER(_i32),
                        ctypes.POINTER(_i32), ctypes.POINTER(_i32)],
     "gs_sketch_coefficients": [_vp, ctypes.POINTER(_u64)],
-    "gs_sketch_insert_passes": [_vp, ctypes.POINTER(_i32), ctypes.POINTER(_i32)],
     "gs_sketch_zero": [_vp, _vp],
     "gs_accumulate": [_vp, _vp, _vp, _i64, _f32, _vp],
     "gs_sketch_insert": [_vp, _i32, _vp, _i64, _vp],
@@ -154,13 +153,6 @@ def gs_sketch_info(sketch: int) -> dict:
                                          ctypes.byref(g), ctypes.byref(rp)), "gs_sketch_info")
     return {"r": r.value, "c": c.value, "workers": w.value, "group_width": g.value,
             "rows_per_pass": rp.value}
-
-
-def gs_sketch_insert_passes(sketch: int) -> dict:
-    n, parts = _i32(), _i32()
-    _check(load_library().gs_sketch_insert_passes(sketch, ctypes.byref(n), ctypes.byref(parts)),
-           "gs_sketch_insert_passes")
-    return {"passes": n.value, "bucket_parts": parts.value}
 
 
 def gs_sketch_coefficients(sketch: int):

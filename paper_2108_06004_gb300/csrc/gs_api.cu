@@ -12,7 +12,6 @@
 struct gs_sketch {
   int32_t r, c, workers, W, groups;
   int32_t rows_per_pass;  // rows inserted per pass of the fused kernel (table slice <= L2 budget)
-  int32_t parts;          // bucket ranges per row when one row exceeds the budget (else 1)
   uint64_t seed;
   gs::HashCoeffs h;
   float* tables;  // groups * r*c*W
@@ -102,33 +101,16 @@ int choose_rows_per_pass(int r, int c, int W) {
   return (int)n;
 }
 
-// A row larger than the pass budget is inserted in this many bucket ranges, one per pass.
-int choose_parts(int c, int W) {
-  const size_t row_bytes = (size_t)c * (size_t)W * sizeof(float);
-  const size_t n = (row_bytes + kPassBudget - 1) / kPassBudget;
-  return n < 1 ? 1 : (int)(n < (size_t)c ? n : (size_t)c);
-}
-
-// The passes of one group's insert: row ranges of rows_per_pass rows, each row split into
-// `parts` bucket ranges when it exceeds the budget.  The first pass also accumulates.
+// The row ranges of one group's insert passes, rows_per_pass rows each; the first pass also
+// accumulates.
 struct Pass {
   int j0, j1;
-  uint32_t blo, bspan;  // bspan 0: every bucket
 };
 
 std::vector<Pass> insert_passes(const gs_sketch* sk) {
   std::vector<Pass> out;
-  if (sk->parts <= 1) {
-    for (int j0 = 0; j0 < sk->r; j0 += sk->rows_per_pass)
-      out.push_back({j0, (j0 + sk->rows_per_pass < sk->r) ? j0 + sk->rows_per_pass : sk->r, 0u, 0u});
-    return out;
-  }
-  for (int j = 0; j < sk->r; ++j) {
-    for (int q = 0; q < sk->parts; ++q) {
-      const uint64_t lo = (uint64_t)sk->c * q / sk->parts, hi = (uint64_t)sk->c * (q + 1) / sk->parts;
-      out.push_back({j, j + 1, (uint32_t)lo, (uint32_t)(hi - lo)});
-    }
-  }
+  for (int j0 = 0; j0 < sk->r; j0 += sk->rows_per_pass)
+    out.push_back({j0, (j0 + sk->rows_per_pass < sk->r) ? j0 + sk->rows_per_pass : sk->r});
   return out;
 }
 
@@ -206,8 +188,6 @@ gs_status accumulate_insert_impl(gs_sketch* sk, int32_t first, int32_t n, float*
     for (const Pass& ps : insert_passes(sk)) {
       p.j0 = ps.j0;
       p.j1 = ps.j1;
-      p.blo = ps.blo;
-      p.bspan = ps.bspan;
       cudaError_t err = gs::launch_accumulate_insert(p, W, first, vec, s);
       if (err != cudaSuccess) return cuda_fail(err, "accumulate_insert launch");
       first = false;
@@ -239,8 +219,6 @@ gs_status insert_all_impl(gs_sketch* sk, const float* const* vec, int64_t d, cud
     for (const Pass& ps : insert_passes(sk)) {
       p.j0 = ps.j0;
       p.j1 = ps.j1;
-      p.blo = ps.blo;
-      p.bspan = ps.bspan;
       cudaError_t err = gs::launch_accumulate_insert(p, W, false, vec_ok, s);
       if (err != cudaSuccess) return cuda_fail(err, "insert launch");
     }
@@ -650,7 +628,6 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
   sk->W = W;
   sk->groups = groups;
   sk->rows_per_pass = choose_rows_per_pass(r, c, W);
-  sk->parts = choose_parts(c, W);
   sk->seed = seed;
   derive_coefficients(r, seed, sk->h);
   sk->tables = mem;
@@ -681,13 +658,6 @@ gs_status gs_sketch_info(const gs_sketch* sk, int32_t* r, int32_t* c, int32_t* w
   if (workers) *workers = sk->workers;
   if (group_width) *group_width = sk->W;
   if (rows_per_pass) *rows_per_pass = sk->rows_per_pass;
-  return GS_OK;
-}
-
-gs_status gs_sketch_insert_passes(const gs_sketch* sk, int32_t* passes, int32_t* bucket_parts) {
-  if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
-  if (passes) *passes = (int32_t)insert_passes(sk).size();
-  if (bucket_parts) *bucket_parts = sk->parts;
   return GS_OK;
 }
 
@@ -1255,8 +1225,6 @@ gs_status gs_insert_request_ceiling(gs_sketch* sk, int64_t d, void* window, size
       if (e != cudaSuccess) break;
       p.j0 = ps.j0;
       p.j1 = ps.j1;
-      p.blo = ps.blo;
-      p.bspan = ps.bspan;
       e = gs::launch_insert_ceiling_probe(p, W, first, s);
       first = false;
     }

@@ -80,7 +80,6 @@ struct InsertParams {
   int32_t lane;      // single-vector insert: the lane written
   int32_t r;
   int32_t j0, j1;    // rows inserted by this launch: [j0, j1)
-  uint32_t blo, bspan;  // and of those rows only buckets b with b - blo < bspan (bspan 0: all)
   uint32_t c, cmask;
   float rho;
   int64_t winmask;   // request-ceiling probe only: vector offsets are taken modulo winmask + 1

@@ -13,9 +13,7 @@
 // G = W/4 adjacent lanes shares one coordinate quad, each lane owns four workers, and one
 // warp instruction writes whole W*4-byte cells with 16-byte vector reductions
 // (red.global.add.v4.f32).  For tables larger than the L2 budget the rows are inserted in
-// passes over row ranges: the first pass accumulates, later passes only re-read e.  A row too
-// large for one pass is split into bucket ranges: each pass then updates only the cells of its
-// range, and every coordinate whose bucket falls elsewhere skips its reduction.
+// passes over row ranges: the first pass accumulates, later passes only re-read e.
 #include "gs_common.cuh"
 
 namespace gs {
@@ -123,7 +121,6 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_const
       }
     }
     const int tmax = (d - i0 < 4) ? (int)(d - i0) : 4;
-    const uint32_t bspan = prm.bspan ? prm.bspan : 0xFFFFFFFFu;
 #pragma unroll 1
     for (int j = prm.j0; j < prm.j1; ++j) {
       const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
@@ -136,9 +133,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert(const __grid_const
           const uint32_t bk = bucket_of<POW2>(x, prm.c, prm.cmask);
           const uint32_t sb = signbit_of(y);
           float* cell = row + (size_t)bk * W;
-          if (bk - prm.blo >= bspan) {
-            // another pass covers this bucket
-          } else if (W == 1) {
+          if (W == 1) {
             red_add_f32(cell, apply_sign(ev[0][t], sb));
           } else {
             red_add_v2(cell, apply_sign(ev[0][t], sb), apply_sign(ev[W > 1 ? 1 : 0][t], sb));
@@ -178,7 +173,6 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_
       }
     }
     const int tmax = (d - i0 < 4) ? (int)(d - i0) : 4;
-    const uint32_t bspan = prm.bspan ? prm.bspan : 0xFFFFFFFFu;
 #pragma unroll 1
     for (int j = prm.j0; j < prm.j1; ++j) {
       const uint64_t a = prm.h.a[j], a2 = prm.h.a2[j];
@@ -190,9 +184,8 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_
         if (t < tmax) {
           const uint32_t bk = bucket_of<POW2>(x, prm.c, prm.cmask);
           const uint32_t sb = signbit_of(y);
-          if (bk - prm.blo < bspan)  // else another pass covers this bucket
-            red_add_v4(row + (size_t)bk * W, apply_sign(ev[0][t], sb), apply_sign(ev[1][t], sb),
-                       apply_sign(ev[2][t], sb), apply_sign(ev[3][t], sb));
+          red_add_v4(row + (size_t)bk * W, apply_sign(ev[0][t], sb), apply_sign(ev[1][t], sb),
+                     apply_sign(ev[2][t], sb), apply_sign(ev[3][t], sb));
           x = step61(x, a);
           y = step61(y, a2);
         }
