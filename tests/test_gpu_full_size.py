@@ -169,4 +169,7 @@ def run_full_size(gs, H, name, steps):
 
 @pytest.mark.parametrize("name,steps", [("resnet18", 5), ("resnet50", 5), ("vgg16", 2), ("bert-large", 2)])
 def test_full_size_steps(gs, H, name, steps):
-    run_full_size(gs, H, name, steps)
+    try:
+        run_full_size(gs, H, name, steps)
+    finally:
+        torch.cuda.empty_cache()   # return the workload's device memory to the driver for later tests
