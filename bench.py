@@ -500,7 +500,8 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
         "timed_phases": ph["n"],
         "timing": "event-record nodes inside the step's CUDA graph" if run.use_plan else "CUDA events around the call",
     }
-    ceil_ms = probes.get("insert_ms")
+    # the probe stands for the fused accumulate + insert; the sketched state inserts raw gradients
+    ceil_ms = probes.get("insert_ms") if variant != "sketched_state" else None
     k1["co_bound"] = {
         "kind": "SM->L2 requests: one cell reduction per (coordinate, row, group) plus the u, e stores and the loads",
         "probe": "gs_insert_request_ceiling: the same kernels, grids, buckets and reductions with every vector access "

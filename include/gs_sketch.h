@@ -148,6 +148,15 @@ gs_status gs_accumulate_insert_staged(gs_sketch* sketch, int32_t first_worker, i
  * order for every cell.  Worker tables are left unchanged. */
 gs_status gs_sketch_merge_tree(gs_sketch* sketch, int32_t P, gs_stream stream);
 
+/* The same tree merge over P separately created sketches, for callers that keep one sketch per
+ * worker (gs_sketch_create with workers = 1): the table of worker 0 of sketches[0..P-1], in that
+ * rank order, is merged by the schedule of gs_sketch_merge_tree into the merged table of
+ * sketches[0] (the table gs_query_topk reads).  sketches is a HOST array of P sketch pointers,
+ * all on the current device.  GS_ERR_MISMATCH unless every sketch shares sketches[0]'s r, c and
+ * seed; GS_ERR_INVALID_ARG for P outside [1, GS_MAX_WORKERS] or a sketch listed twice.  The
+ * worker tables are left unchanged. */
+gs_status gs_sketch_merge_sketches(gs_sketch* const* sketches, int32_t P, gs_stream stream);
+
 /* ---- steps 4-5: median query and top-k ------------------------------------------- */
 
 /* Device workspace bytes gs_query_topk needs for d coordinates and k selected. */

@@ -46,6 +46,7 @@ SIGNATURES = {
     "gs_accumulate_insert": [_vp, _i32, _i32, _PP, _PP, _PP, _i64, _f32, _vp],
     "gs_accumulate_insert_staged": [_vp, _i32, _i32, _PP, _PP, _PP, _i64, _f32, _vp],
     "gs_sketch_merge_tree": [_vp, _i32, _vp],
+    "gs_sketch_merge_sketches": [_PP, _i32, _vp],
     "gs_query_topk_workspace_size": [_i64, _i64, ctypes.POINTER(_sz)],
     "gs_query_topk": [_vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp],
     "gs_query_topk_noalloc": [_vp, _i64, _i64, _vp, _vp, _vp],
@@ -196,6 +197,12 @@ def gs_accumulate_insert_staged(sketch: int, first_worker: int, momentum, error,
 
 def gs_sketch_merge_tree(sketch: int, P: int, stream=None) -> None:
     _check(load_library().gs_sketch_merge_tree(sketch, P, _stream(stream)), "gs_sketch_merge_tree")
+
+
+def gs_sketch_merge_sketches(sketches, stream=None) -> None:
+    """Tree merge of separately created sketches into the merged table of sketches[0]."""
+    arr = (ctypes.c_void_p * len(sketches))(*sketches)
+    _check(load_library().gs_sketch_merge_sketches(arr, len(sketches), _stream(stream)), "gs_sketch_merge_sketches")
 
 
 def gs_query_topk_workspace_size(d: int, k: int) -> int:

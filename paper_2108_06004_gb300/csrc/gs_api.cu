@@ -792,6 +792,32 @@ gs_status gs_sketch_merge_tree(gs_sketch* sk, int32_t P, gs_stream stream) {
   return GS_OK;
 }
 
+gs_status gs_sketch_merge_sketches(gs_sketch* const* sketches, int32_t P, gs_stream stream) {
+  GS_GUARD_BEGIN
+  if (!sketches) return fail(GS_ERR_INVALID_ARG, "sketches is NULL");
+  if (P < 1 || P > GS_MAX_WORKERS) return fail(GS_ERR_INVALID_ARG, "P must lie in [1, 64]");
+  for (int i = 0; i < P; ++i) {
+    GS_TRY(check_sketch(sketches[i]));
+    if (!same_family(sketches[0], sketches[i]))
+      return fail(GS_ERR_MISMATCH, "sketch " + std::to_string(i) + " differs from sketch 0 in r, c or seed");
+    for (int j = 0; j < i; ++j)
+      if (sketches[j] == sketches[i]) return fail(GS_ERR_INVALID_ARG, "a sketch appears twice");
+  }
+  gs::MergeListParams mp;
+  std::memset(&mp, 0, sizeof(mp));
+  for (int i = 0; i < P; ++i) {
+    mp.tables[i] = sketches[i]->tables;
+    mp.lane_stride[i] = sketches[i]->W;
+  }
+  mp.merged = sketches[0]->merged;
+  mp.cells = (int64_t)sketches[0]->r * sketches[0]->c;
+  mp.P = P;
+  cudaError_t e = gs::launch_merge_list(mp, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+  return GS_OK;
+  GS_GUARD_END
+}
+
 gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes) {
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");

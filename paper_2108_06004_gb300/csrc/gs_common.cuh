@@ -94,6 +94,14 @@ struct MergeParams {
   int32_t P;
 };
 
+struct MergeListParams {
+  const float* tables[GS_MAX_WORKERS];   // worker 0's table of each sketch, [r][c][lane_stride]
+  int32_t lane_stride[GS_MAX_WORKERS];
+  float* merged;                          // [r][c]
+  int64_t cells;
+  int32_t P;
+};
+
 struct GatherParams {
   float* u[GS_MAX_WORKERS];
   float* e[GS_MAX_WORKERS];
@@ -130,6 +138,7 @@ cudaError_t launch_insert_staged(const InsertParams& p, int W, cudaStream_t s);
 cudaError_t launch_hash_eval(const HashCoeffs& h, int r, uint32_t c, const int64_t* coords,
                              int64_t n, int32_t* bucket_out, int8_t* sign_out, cudaStream_t s);
 cudaError_t launch_merge(const MergeParams& p, int W, cudaStream_t s);
+cudaError_t launch_merge_list(const MergeListParams& p, cudaStream_t s);
 cudaError_t launch_gather_and_zero(const GatherParams& p, cudaStream_t s);
 cudaError_t launch_apply_update(float* w, int64_t d, const int64_t* idx, const float* vals, int64_t k, float lr,
                                 cudaStream_t s);

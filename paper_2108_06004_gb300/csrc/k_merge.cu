@@ -70,6 +70,39 @@ __global__ void __launch_bounds__(kBlock) k_merge(const __grid_constant__ MergeP
   }
 }
 
+// The same tree over P separately allocated tables: cell q of input i is
+// tables[i][q * lane_stride[i]] (worker 0 of a sketch whose tables interleave lane_stride
+// workers).
+template <int PMAX>
+__global__ void __launch_bounds__(kBlock) k_merge_list(const __grid_constant__ MergeListParams prm) {
+  grid_begin();
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int P = prm.P;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < prm.cells; q += stride) {
+    float v[PMAX];
+#pragma unroll
+    for (int i = 0; i < PMAX; ++i) v[i] = i < P ? __ldcs(prm.tables[i] + q * prm.lane_stride[i]) : 0.f;
+#pragma unroll
+    for (int s = 1; s < PMAX; s *= 2) {
+#pragma unroll
+      for (int a = 0; a + s < PMAX; a += 2 * s) {
+        if (a + s < P) v[a] = __fadd_rn(v[a + s], v[a]);  // sends = recvs + sends
+      }
+    }
+    prm.merged[q] = v[0];
+  }
+}
+
+template <int PMAX>
+cudaError_t launch_list_t(const MergeListParams& p, cudaStream_t s) {
+  auto kern = k_merge_list<PMAX>;
+  const int64_t need = (p.cells + kBlock - 1) / kBlock;
+  const int64_t cap = (int64_t)device_info().sms * blocks_per_sm((const void*)kern, kBlock);
+  const int grid = (int)(need < 1 ? 1 : (need < cap ? need : cap));
+  launch(kern, grid, kBlock, s, p);
+  return cudaGetLastError();
+}
+
 template <int W, int PMAX>
 cudaError_t launch_t(const MergeParams& p, cudaStream_t s) {
   auto kern = k_merge<W, PMAX>;
@@ -91,6 +124,16 @@ cudaError_t launch_w(const MergeParams& p, cudaStream_t s) {
 }
 
 }  // namespace
+
+cudaError_t launch_merge_list(const MergeListParams& p, cudaStream_t s) {
+  if (p.P <= 1) return launch_list_t<1>(p, s);
+  if (p.P <= 2) return launch_list_t<2>(p, s);
+  if (p.P <= 4) return launch_list_t<4>(p, s);
+  if (p.P <= 8) return launch_list_t<8>(p, s);
+  if (p.P <= 16) return launch_list_t<16>(p, s);
+  if (p.P <= 32) return launch_list_t<32>(p, s);
+  return launch_list_t<64>(p, s);
+}
 
 cudaError_t launch_merge(const MergeParams& p, int W, cudaStream_t s) {
   switch (W) {

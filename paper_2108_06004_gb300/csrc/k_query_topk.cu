@@ -299,91 +299,6 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
   }
 }
 
-// Software-pipelined form of k_query (same results): the rows that bound the median (the first
-// r/2 + 1) of the thread's next quad are loaded together with the remaining rows of its current
-// quad, so that one round trip to L2 serves both.
-template <int R>
-__global__ void __launch_bounds__(kBlock) k_query_pipe(const __grid_constant__ QueryParams prm) {
-  grid_begin();
-  __shared__ uint32_t sh[kBins];
-  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
-  __syncthreads();
-  const int64_t d = prm.d, nq = (d + 3) / 4;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  const int lane = threadIdx.x & 31;
-  const uint32_t pk = prune_key_of(prm);
-  constexpr int kF = R / 2 + 1;  // rows that bound the median
-  float head[4][kF];
-  auto load_head = [&](int64_t q) {
-    const int64_t i0 = q * 4;
-    const int tmax = q < nq ? (d - i0 < 4 ? (int)(d - i0) : 4) : 0;
-#pragma unroll
-    for (int j = 0; j < kF; ++j) {
-      uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
-      uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
-      const float* row = prm.T + (size_t)j * prm.c;
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        head[t][j] = 0.f;
-        if (t < tmax) {
-          head[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
-          x = step61(x, prm.h.a[j]);
-          y = step61(y, prm.h.a2[j]);
-        }
-      }
-    }
-  };
-  int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31);
-  if (q0 < nq) load_head(q0 + lane);
-  for (; q0 < nq; q0 += stride) {
-    const int64_t q = q0 + lane;
-    const int64_t i0 = q * 4;
-    const int tmax = q < nq ? (d - i0 < 4 ? (int)(d - i0) : 4) : 0;
-    float v[4][R];
-    bool need[4];
-#pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      bool below = pk != 0u;
-#pragma unroll
-      for (int j = 0; j < kF; ++j) {
-        v[t][j] = head[t][j];
-        below = below && key_of(v[t][j]) < pk;
-      }
-      need[t] = !below;
-    }
-#pragma unroll
-    for (int j = kF; j < R; ++j) {
-      uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
-      uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
-      const float* row = prm.T + (size_t)j * prm.c;
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        v[t][j] = 0.f;
-        if (t < tmax) {
-          if (need[t]) v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
-          x = step61(x, prm.h.a[j]);
-          y = step61(y, prm.h.a2[j]);
-        }
-      }
-    }
-    if (q0 + stride < nq) load_head(q0 + stride + lane);  // warp-uniform; in flight with the rows above
-    float m[4] = {0.f, 0.f, 0.f, 0.f};
-    if (tmax > 0) {
-#pragma unroll
-      for (int t = 0; t < 4; ++t) m[t] = need[t] ? median_of<R>(v[t]) : __uint_as_float(kPrunedBits);
-      store_est(prm, i0, tmax, m);
-    }
-    if (prm.hist_on) {
-#pragma unroll
-      for (int t = 0; t < 4; ++t) hist_add(sh, t < tmax ? (key_of(m[t]) >> kL1Shift) : kNone);
-    }
-  }
-  if (prm.hist_on) {
-    hist_flush(sh, prm.hist, kBins);
-    last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
-  }
-}
-
 // Runs after k_query.  If the level-1 pick landed in the prune key's bin or above, the k-th
 // largest |est| is at least the prune key and pruning changed nothing the selection sees: the
 // kernel returns at once.  Otherwise every stored -0.0 (each pruned coordinate, and any
@@ -1091,12 +1006,9 @@ int persistent_grid(K kernel, int64_t work_items, int block) {
   return (int)(need < 1 ? 1 : (need < cap ? need : cap));
 }
 
-// Which form of the fast-path query runs (both give the same estimate and selection).
-constexpr bool kQueryPipelined = false;
-
 template <int R>
 cudaError_t launch_query_r(const QueryParams& p, cudaStream_t s) {
-  auto kern = kQueryPipelined ? k_query_pipe<R> : k_query<R>;
+  auto kern = k_query<R>;
   launch(kern, persistent_grid(kern, (p.d + 3) / 4, kBlock), kBlock, s, p);
   return cudaGetLastError();
 }

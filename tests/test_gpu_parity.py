@@ -204,6 +204,44 @@ def test_accumulate_insert_staged_rejects_large_rows(gs, H):
         run.close()
 
 
+@pytest.mark.parametrize("P,d,r,c", [(1, 10_007, 3, 512), (5, 100_003, 5, 4096), (13, 50_001, 4, 1000), (64, 20_011, 3, 256)])
+def test_merge_separate_sketches(gs, H, P, d, r, c):
+    """P sketches created one per worker (the problem statement's form of the merge): the merged
+    table of sketches[0] is bit-equal to the fp32 tree of their tables in the schedule's order and
+    within 1e-5*A of the oracle's fp64 tree of the workers' sketches; mismatched families and a
+    repeated sketch are rejected."""
+    seed = 900 + P
+    rng = np.random.default_rng(seed)
+    coeffs = oracle.derive_coefficients(r, seed)
+    sks = [gs.gs_sketch_create(r, c, seed, 1, 0) for _ in range(P)]
+    other = gs.gs_sketch_create(r, c, seed + 1, 1, 0)
+    try:
+        xs = [(rng.standard_normal(d) * 1e-3).astype(np.float32) for _ in range(P)]
+        for sk, x in zip(sks, xs):
+            gs.gs_sketch_insert(sk, 0, _dev(x), d)
+        gs.gs_sketch_merge_sketches(sks)
+        tabs = []
+        for sk in sks:
+            buf = np.empty(r * c, np.float32)
+            gs.gs_sketch_copy_to_host(sk, 0, buf)
+            tabs.append(buf.reshape(r, c))
+        merged = np.empty(r * c, np.float32)
+        gs.gs_sketch_copy_to_host(sks[0], -1, merged)
+        assert np.array_equal(merged.reshape(r, c), H.fp32_tree(tabs))
+        ors = [oracle.sketch(x, coeffs, c) for x in xs]
+        H.check_cells(merged.reshape(r, c), oracle.merge_tree([t for t, _ in ors]),
+                      oracle.merge_tree([a for _, a in ors]), "merged")
+        with pytest.raises(gs.GsError) as ei:
+            gs.gs_sketch_merge_sketches(sks[:1] + [other])
+        assert ei.value.status == gs.GS_ERR_MISMATCH
+        with pytest.raises(gs.GsError) as ei:
+            gs.gs_sketch_merge_sketches([sks[0], sks[0]])
+        assert ei.value.status == gs.GS_ERR_INVALID_ARG
+    finally:
+        for sk in sks + [other]:
+            gs.gs_sketch_destroy(sk)
+
+
 def test_accumulate_insert_unaligned(gs, H):
     """Vectors that start 4 bytes past a 16-byte boundary take the scalar load path of the
     fused kernel; the state stays bit-exact and the tables agree with the oracle."""
