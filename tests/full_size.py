@@ -10,10 +10,11 @@ here exactly as ``oracle.step`` computes it, piece by piece:
 
   * the hash buckets and signs of all d coordinates, once per test, into files that every
     process maps (``hash_rows`` per piece);
-  * per worker, one task: ``accumulate`` piece by piece from the GPU's pre-step state and the
-    step's gradient, the bit-exact comparison with the GPU's post-step momentum and error
-    (zero at the selected coordinates), and the worker's fp64 sketch and magnitude table
-    summed over the pieces; also the accumulated error at the selected coordinates;
+  * per worker, tasks over parts of its pieces (so that every process is busy): ``accumulate``
+    piece by piece from the GPU's pre-step state and the step's gradient, the bit-exact
+    comparison with the GPU's post-step momentum and error (zero at the selected coordinates),
+    and the worker's fp64 sketch and magnitude table summed over the pieces; also the
+    accumulated error at the selected coordinates;
   * ``merge_tree`` of the worker tables (in the calling process);
   * the median query and its tolerance band, piece by piece into mapped files.
 
@@ -57,9 +58,12 @@ def _hash_task(args):
 
 
 def _worker_task(args):
-    """One worker's step from its slot of mapped vectors (u0, e0, g: the GPU's state before the
-    step and the step's gradient; ug, eg: the GPU's state after it)."""
-    dirpath, slot, coeffs, c, d, rho, sel = args
+    """One worker's step, over the pieces [p0, p1) of its coordinate range, from its slot of
+    mapped vectors (u0, e0, g: the GPU's state before the step and the step's gradient; ug, eg:
+    the GPU's state after it).  Returns the fp64 sketch and magnitude table of those pieces, the
+    accumulated error at the selected coordinates inside them (zero elsewhere), and the counts of
+    momentum / error values that differ from the GPU's and of selected values not zeroed."""
+    dirpath, slot, coeffs, c, d, rho, sel, p0, p1 = args
     bk = _mapped(os.path.join(dirpath, "buckets.npy"), None, None, "r")
     sg = _mapped(os.path.join(dirpath, "signs.npy"), None, None, "r")
     vec = {n: _mapped(os.path.join(dirpath, f"slot{slot}_{n}.npy"), None, None, "r")
@@ -69,7 +73,7 @@ def _worker_task(args):
     A = np.zeros((r, c))
     e_sel = np.zeros(sel.size, np.float32)
     bad_u = bad_e = nonzero_sel = 0
-    for a, b in _pieces(d):
+    for a, b in _pieces(d)[p0:p1]:
         u1, e1 = oracle.accumulate(vec["u0"][a:b], vec["e0"][a:b], vec["g"][a:b], rho)
         lo, hi = np.searchsorted(sel, [a, b])
         loc = sel[lo:hi] - a
@@ -148,10 +152,23 @@ class ParallelOracle:
         return _mapped(self.slot_path(slot, name), None, None, "r+")
 
     def workers(self, slot_ids, rho: float, sel):
-        """Run the worker tasks of the filled slots; returns their results in slot order."""
+        """Run the worker tasks of the filled slots, each slot's pieces split over enough tasks
+        to keep every process busy; returns one combined result per slot, in slot order."""
         sel = np.ascontiguousarray(np.sort(np.asarray(sel, np.int64)))
-        return self.pool.map(_worker_task, [(self.dir, s, self.coeffs, self.c, self.d, rho, sel) for s in slot_ids],
-                             chunksize=1)
+        slot_ids = list(slot_ids)
+        npieces = len(_pieces(self.d))
+        split = max(1, min(npieces, -(-self.procs // max(1, len(slot_ids)))))
+        bounds = [(npieces * q // split, npieces * (q + 1) // split) for q in range(split)]
+        tasks = [(self.dir, s, self.coeffs, self.c, self.d, rho, sel, p0, p1) for s in slot_ids for p0, p1 in bounds]
+        parts = self.pool.map(_worker_task, tasks, chunksize=1)
+        out = []
+        for n in range(len(slot_ids)):
+            mine = parts[n * split:(n + 1) * split]
+            T = sum(m[0] for m in mine)
+            A = sum(m[1] for m in mine)
+            e_sel = sum(m[2] for m in mine)
+            out.append((T, A, e_sel, sum(m[3] for m in mine), sum(m[4] for m in mine), sum(m[5] for m in mine)))
+        return out
 
     def query(self, merged, merged_abs, rel: float = 1e-5):
         """(est, band): the fp64 median estimate of every coordinate and its tolerance band."""

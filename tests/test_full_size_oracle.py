@@ -34,6 +34,10 @@ def test_parallel_oracle_equals_plain_step(monkeypatch):
         assert np.allclose(est, res.est, rtol=0, atol=1e-12)
         assert np.allclose(band, oracle.cell_band(res.merged_abs, co, np.arange(d)), rtol=1e-13, atol=0)
         assert np.array_equal(oracle.topk_by_threshold(est, k), res.idx)
+        # one slot alone is split over both processes: the same result
+        T0, A0, e0, bu0, be0, nz0 = po.workers([0], rho, res.idx)[0]
+        assert np.allclose(T0, out[0][0], rtol=0, atol=1e-12 * res.abs_tables[0].max())
+        assert np.array_equal(e0, out[0][2]) and bu0 == be0 == nz0 == 0
         # a planted mistake in the GPU-side state is counted
         po.slot(0, "eg")[5] = np.float32(1.0)
         assert po.workers([0], rho, res.idx)[0][4] == 1
