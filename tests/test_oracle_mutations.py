@@ -77,7 +77,8 @@ def test_pin_catches_mutation(monkeypatch, name, bad, pin, kw):
 # ---- the later oracle functions (weight update, HEAVYMIX, sketched state) -----------------
 
 _REAL = {n: getattr(gssgd, n) for n in ("apply_update", "gather_and_zero", "heavymix_select",
-                                         "sketched_state_step", "merge_schedule")}
+                                         "sketched_state_step", "merge_schedule", "sketch",
+                                         "heavymix_select_from")}
 _REAL["derive_coefficients"] = cs.derive_coefficients
 _REAL["splitmix64_at"] = cs.splitmix64_at
 
@@ -141,7 +142,41 @@ def _sketched_state_error_from_s(U, E, AU, AE, gs, rho, coeffs, c, k, rel=1e-5):
     return res
 
 
+def _topk_threshold_ties_high(est, k):
+    a = np.abs(np.asarray(est, dtype=np.float64))
+    tau = np.partition(a, a.size - k)[a.size - k]
+    gt = np.nonzero(a > tau)[0]
+    eq = np.nonzero(a == tau)[0]
+    return np.sort(np.concatenate([gt, eq[eq.size - (k - gt.size):]])).astype(np.int64)  # larger indices
+
+
+def _sketch_ignores_global_coordinates(x, coeffs, c, hashes=None, idx=None):
+    return _REAL["sketch"](x, coeffs, c, hashes)       # every piece hashed at 0 .. len - 1
+
+
+def _heavymix_members_strict(est, l2sq, k):
+    est = np.asarray(est, dtype=np.float64)
+    return est * est > l2sq / k                          # > in place of >=
+
+
+def _heavymix_fill_largest_xi(in_h, est, k, fill_seed):
+    in_h = np.asarray(in_h, dtype=bool)
+    if int(in_h.sum()) >= k:
+        return _REAL["heavymix_select_from"](in_h, est, k, fill_seed)
+    NH = np.nonzero(~in_h)[0]
+    xi = (cs.splitmix64_at(fill_seed, NH) >> np.uint64(33)).astype(np.int64)
+    fill = NH[np.lexsort((NH, -xi))[: k - int(in_h.sum())]]   # largest xi first
+    return np.sort(np.concatenate([np.nonzero(in_h)[0], fill])).astype(np.int64)
+
+
 LATER = [
+    ("topk_by_threshold", _topk_threshold_ties_high, pins.test_topk_by_threshold_equals_topk, {}),
+    ("sketch", _sketch_ignores_global_coordinates, pins.test_sketch_in_pieces_equals_whole, {}),
+    ("heavymix_members", _heavymix_members_strict, pins.test_heavymix_select_brute_force_threshold_on_the_square,
+     {}),
+    ("heavymix_select_from", _heavymix_fill_largest_xi, pins.test_heavymix_select_brute_force_threshold_on_the_square,
+     {}),
+    ("heavymix_select_from", _heavymix_fill_largest_xi, pins.test_heavymix_random_fill_brute_force, {}),
     ("apply_update", _apply_update_fused, pins.test_apply_update_equals_numpy_fp32, {}),
     ("apply_update", _apply_update_ascent, pins.test_apply_update_closed_form, {}),
     ("gather_and_zero", _gather_keeps_momentum, pins.test_gather_and_zero_conservation, {}),

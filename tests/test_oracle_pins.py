@@ -440,7 +440,10 @@ def test_heavymix_select_brute_force_threshold_on_the_square():
     and the fill by (xi_i, i) over the rest."""
     est = np.array([3.0, -2.0, 1.9, 2.5, -0.7, 0.1, 4.5, -3.9, 0.05, 1.0, -2.1, 0.3])
     d = est.size
-    for k, l2sq, seed in [(3, 12.0, 0), (4, 16.0, 9), (5, 20.0, 77), (2, 8.0, 2**64 - 5), (6, 3.0, 1)]:
+    # |H| >= k (top-k of H) and |H| < k (H plus the fill), with est_i^2 exactly at the threshold
+    # for i = 1 (l2sq / k = 4) in several of them
+    for k, l2sq, seed in [(3, 12.0, 0), (4, 16.0, 9), (5, 20.0, 77), (2, 8.0, 2**64 - 5), (6, 3.0, 1),
+                          (8, 32.0, 5), (10, 40.0, 12345), (9, 36.0, 2**63), (11, 176.0, 7), (12, 1e6, 3)]:
         thr = l2sq / k
         h = [i for i in range(d) if est[i] * est[i] >= thr]
         if len(h) >= k:
