@@ -59,7 +59,7 @@ def accumulate(u: np.ndarray, e: np.ndarray, g: np.ndarray, rho: float):
 # ---- 2. sketch -------------------------------------------------------------------------
 
 def sketch(x: np.ndarray, coeffs, c: int, hashes=None, idx=None):
-    """Count Sketch of vector x: (T, A), both [r, c] fp64.
+    """Count Sketch of vector x (fp32, or an fp64 sum of fp32 vectors): (T, A), both [r, c] fp64.
 
     T[j][b] = sum over i with h_j(i) = b of s_j(i) * x_i
     A[j][b] = sum over the same i of |x_i|       (the magnitude carried by the cell)
@@ -69,7 +69,7 @@ def sketch(x: np.ndarray, coeffs, c: int, hashes=None, idx=None):
     at its own global coordinates.  ``hashes`` may pass ``hash_rows(coeffs, c, idx)`` computed
     once for many vectors.
     """
-    x64 = np.asarray(x, dtype=np.float32).astype(np.float64)
+    x64 = np.asarray(x, dtype=np.float64)     # fp32 vectors widen exactly; fp64 sums stay as they are
     d = x64.size
     if hashes is None:
         gi = np.arange(d, dtype=np.uint64) if idx is None else np.asarray(idx, dtype=np.uint64)

@@ -10,12 +10,15 @@ here exactly as ``oracle.step`` computes it, piece by piece:
 
   * the hash buckets and signs of all d coordinates, once per test, into files that every
     process maps (``hash_rows`` per piece);
-  * per worker, tasks over parts of its pieces (so that every process is busy): ``accumulate``
-    piece by piece from the GPU's pre-step state and the step's gradient, the bit-exact
-    comparison with the GPU's post-step momentum and error (zero at the selected coordinates),
-    and the worker's fp64 sketch and magnitude table summed over the pieces; also the
-    accumulated error at the selected coordinates;
-  * ``merge_tree`` of the worker tables (in the calling process);
+  * for each group of workers held in the slots, tasks over parts of the pieces (so that every
+    process is busy): per worker ``accumulate`` piece by piece from the GPU's pre-step state and
+    the step's gradient, the bit-exact comparison with the GPU's post-step momentum and error
+    (zero at the selected coordinates), the accumulated error at the selected coordinates, and,
+    for the workers asked for, their own fp64 sketch and magnitude table;
+  * the merged table: ``merge_tree`` of the worker tables where every worker has one, else, by
+    the same linearity (pinned: the merge of sketches is the sketch of the sum, and likewise for
+    the magnitude tables), the sketch of the fp64 sum of the workers' accumulated error vectors
+    and the magnitude table of the sum of their absolute values;
   * the median query and its tolerance band, piece by piece into mapped files.
 
 The pool is started with the "spawn" method, so that no child inherits a CUDA context.
@@ -57,37 +60,50 @@ def _hash_task(args):
     return b - a
 
 
-def _worker_task(args):
-    """One worker's step, over the pieces [p0, p1) of its coordinate range, from its slot of
-    mapped vectors (u0, e0, g: the GPU's state before the step and the step's gradient; ug, eg:
-    the GPU's state after it).  Returns the fp64 sketch and magnitude table of those pieces, the
-    accumulated error at the selected coordinates inside them (zero elsewhere), and the counts of
-    momentum / error values that differ from the GPU's and of selected values not zeroed."""
-    dirpath, slot, coeffs, c, d, rho, sel, p0, p1 = args
+def _group_task(args):
+    """A group of workers' step over the pieces [p0, p1) of the coordinate range, from their
+    slots of mapped vectors (u0, e0, g: the GPU's state before the step and the step's gradient;
+    ug, eg: the GPU's state after it).  Per worker: the accumulated error at the selected
+    coordinates inside those pieces (zero elsewhere) and the counts of momentum / error values
+    that differ from the GPU's and of selected values not zeroed; for the workers in `tabled`,
+    their own fp64 sketch and magnitude table.  For the group: the sketch of the sum of its
+    accumulated error vectors and the magnitude table of the sum of their absolute values (by
+    linearity, their merge)."""
+    dirpath, slots, tabled, coeffs, c, d, rho, sel, p0, p1 = args
     bk = _mapped(os.path.join(dirpath, "buckets.npy"), None, None, "r")
     sg = _mapped(os.path.join(dirpath, "signs.npy"), None, None, "r")
-    vec = {n: _mapped(os.path.join(dirpath, f"slot{slot}_{n}.npy"), None, None, "r")
-           for n in ("u0", "e0", "g", "ug", "eg")}
     r = bk.shape[0]
-    T = np.zeros((r, c))
-    A = np.zeros((r, c))
-    e_sel = np.zeros(sel.size, np.float32)
-    bad_u = bad_e = nonzero_sel = 0
+    vecs = {s: {n: _mapped(os.path.join(dirpath, f"slot{s}_{n}.npy"), None, None, "r")
+                for n in ("u0", "e0", "g", "ug", "eg")} for s in slots}
+    own = {s: (np.zeros((r, c)), np.zeros((r, c))) for s in tabled}
+    T_sum, A_sum = np.zeros((r, c)), np.zeros((r, c))
+    e_sel = {s: np.zeros(sel.size, np.float32) for s in slots}
+    counts = {s: [0, 0, 0] for s in slots}
     for a, b in _pieces(d)[p0:p1]:
-        u1, e1 = oracle.accumulate(vec["u0"][a:b], vec["e0"][a:b], vec["g"][a:b], rho)
+        hashes = (np.asarray(bk[:, a:b]), np.asarray(sg[:, a:b]))
         lo, hi = np.searchsorted(sel, [a, b])
         loc = sel[lo:hi] - a
-        e_sel[lo:hi] = e1[loc]
         keep = np.ones(b - a, bool)
         keep[loc] = False
-        ug, eg = np.asarray(vec["ug"][a:b]), np.asarray(vec["eg"][a:b])
-        bad_u += int(np.count_nonzero(ug[keep].view(np.uint32) != u1[keep].view(np.uint32)))
-        bad_e += int(np.count_nonzero(eg[keep].view(np.uint32) != e1[keep].view(np.uint32)))
-        nonzero_sel += int(np.count_nonzero(ug[loc]) + np.count_nonzero(eg[loc]))
-        t, m = oracle.sketch(e1, coeffs, c, hashes=(np.asarray(bk[:, a:b]), np.asarray(sg[:, a:b])))
-        T += t
-        A += m
-    return T, A, e_sel, bad_u, bad_e, nonzero_sel
+        x_sum = np.zeros(b - a)
+        a_sum = np.zeros(b - a)
+        for s in slots:
+            v = vecs[s]
+            u1, e1 = oracle.accumulate(v["u0"][a:b], v["e0"][a:b], v["g"][a:b], rho)
+            e_sel[s][lo:hi] = e1[loc]
+            ug, eg = np.asarray(v["ug"][a:b]), np.asarray(v["eg"][a:b])
+            counts[s][0] += int(np.count_nonzero(ug[keep].view(np.uint32) != u1[keep].view(np.uint32)))
+            counts[s][1] += int(np.count_nonzero(eg[keep].view(np.uint32) != e1[keep].view(np.uint32)))
+            counts[s][2] += int(np.count_nonzero(ug[loc]) + np.count_nonzero(eg[loc]))
+            x_sum += e1
+            a_sum += np.abs(e1.astype(np.float64))
+            if s in own:
+                t, m = oracle.sketch(e1, coeffs, c, hashes=hashes)
+                own[s][0][:] += t
+                own[s][1][:] += m
+        T_sum += oracle.sketch(x_sum, coeffs, c, hashes=hashes)[0]
+        A_sum += oracle.sketch(a_sum, coeffs, c, hashes=hashes)[1]
+    return T_sum, A_sum, own, e_sel, counts
 
 
 def _query_task(args):
@@ -151,24 +167,27 @@ class ParallelOracle:
     def slot(self, slot: int, name: str) -> np.ndarray:
         return _mapped(self.slot_path(slot, name), None, None, "r+")
 
-    def workers(self, slot_ids, rho: float, sel):
-        """Run the worker tasks of the filled slots, each slot's pieces split over enough tasks
-        to keep every process busy; returns one combined result per slot, in slot order."""
+    def workers(self, slot_ids, rho: float, sel, tabled=()):
+        """The step of the workers in the filled slots, their pieces split over every process.
+        Returns (T_sum, A_sum, own, e_sel, counts): the sketch of the sum of their accumulated
+        error vectors and the magnitude table of the sum of their absolute values; own[slot] =
+        (T, A) for the slots in `tabled`; e_sel[slot], the accumulated error at the selected
+        coordinates; counts[slot] = (momentum values differing from the GPU's, error values
+        differing, selected values not zeroed)."""
         sel = np.ascontiguousarray(np.sort(np.asarray(sel, np.int64)))
         slot_ids = list(slot_ids)
+        tabled = [s for s in slot_ids if s in set(tabled)]
         npieces = len(_pieces(self.d))
-        split = max(1, min(npieces, -(-self.procs // max(1, len(slot_ids)))))
+        split = max(1, min(npieces, self.procs))
         bounds = [(npieces * q // split, npieces * (q + 1) // split) for q in range(split)]
-        tasks = [(self.dir, s, self.coeffs, self.c, self.d, rho, sel, p0, p1) for s in slot_ids for p0, p1 in bounds]
-        parts = self.pool.map(_worker_task, tasks, chunksize=1)
-        out = []
-        for n in range(len(slot_ids)):
-            mine = parts[n * split:(n + 1) * split]
-            T = sum(m[0] for m in mine)
-            A = sum(m[1] for m in mine)
-            e_sel = sum(m[2] for m in mine)
-            out.append((T, A, e_sel, sum(m[3] for m in mine), sum(m[4] for m in mine), sum(m[5] for m in mine)))
-        return out
+        parts = self.pool.map(_group_task, [(self.dir, slot_ids, tabled, self.coeffs, self.c, self.d, rho, sel, p0, p1)
+                                            for p0, p1 in bounds], chunksize=1)
+        T_sum = sum(m[0] for m in parts)
+        A_sum = sum(m[1] for m in parts)
+        own = {s: (sum(m[2][s][0] for m in parts), sum(m[2][s][1] for m in parts)) for s in tabled}
+        e_sel = {s: sum(m[3][s] for m in parts) for s in slot_ids}
+        counts = {s: [sum(m[4][s][q] for m in parts) for q in range(3)] for s in slot_ids}
+        return T_sum, A_sum, own, e_sel, counts
 
     def query(self, merged, merged_abs, rel: float = 1e-5):
         """(est, band): the fp64 median estimate of every coordinate and its tolerance band."""

@@ -284,9 +284,16 @@ def test_merge_of_sketches_is_sketch_of_sum():
     r, c, d, P = 5, 256, 4000, 6
     co = oracle.derive_coefficients(r, 12)
     xs = [_dyadic(rng, d, -64, 64, 2.0**-6) for _ in range(P)]
-    merged = oracle.merge_tree([oracle.sketch(x, co, c)[0] for x in xs])
+    sk = [oracle.sketch(x, co, c) for x in xs]
+    merged = oracle.merge_tree([t for t, _ in sk])
     total = np.sum(np.stack(xs).astype(np.float64), axis=0).astype(np.float32)
     assert np.array_equal(merged, oracle.sketch(total, co, c)[0])
+    # the same with the fp64 sum itself, and the magnitude tables: the merge of the workers'
+    # magnitude tables is the magnitude table of sum_p |x_p|
+    total64 = np.sum(np.stack(xs).astype(np.float64), axis=0)
+    assert np.array_equal(merged, oracle.sketch(total64, co, c)[0])
+    abs64 = np.sum(np.abs(np.stack(xs).astype(np.float64)), axis=0)
+    assert np.array_equal(oracle.merge_tree([a for _, a in sk]), oracle.sketch(abs64, co, c)[1])
 
 
 # ---- top-k -------------------------------------------------------------------------------
