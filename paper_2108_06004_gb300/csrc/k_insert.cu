@@ -13,7 +13,9 @@
 // G = W/4 adjacent lanes shares one coordinate quad, each lane owns four workers, and one
 // warp instruction writes whole W*4-byte cells with 16-byte vector reductions
 // (red.global.add.v4.f32).  For tables larger than the L2 budget the rows are inserted in
-// passes over row ranges: the first pass accumulates, later passes only re-read e.
+// passes over row ranges: the first pass accumulates, later passes only re-read e.  The
+// streams carry an evict_first and the reductions an evict_last L2 policy, so that the table
+// slice of a pass stays in L2 while the vectors flow past it.
 #include "gs_common.cuh"
 
 namespace gs {
@@ -98,6 +100,32 @@ __device__ __forceinline__ void load_lane(const InsertParams& prm, int w, int64_
   }
 }
 
+// load_lane with L2 eviction priorities on the vector streams (the coop kernel's form).
+template <bool ACC, bool VEC, bool WIN>
+__device__ __forceinline__ void load_lane_hinted(const InsertParams& prm, int w, int64_t i0, int64_t d,
+                                                 float (&ev)[4], uint64_t pol) {
+  if (VEC && i0 + 4 <= d) {
+    const int64_t ia = WIN ? (i0 & prm.winmask) : i0;
+    float4 e4 = ld_stream(prm.e[w] + ia, pol);
+    if (ACC) {
+      const float4 g4 = ld_stream(prm.g[w] + ia, pol);
+      float4 u4 = ld_stream(prm.u[w] + ia, pol);
+      acc1(prm.rho, u4.x, e4.x, g4.x);
+      acc1(prm.rho, u4.y, e4.y, g4.y);
+      acc1(prm.rho, u4.z, e4.z, g4.z);
+      acc1(prm.rho, u4.w, e4.w, g4.w);
+      st_stream(prm.u[w] + ia, u4, pol);
+      st_stream(prm.e[w] + ia, e4, pol);
+    }
+    ev[0] = e4.x;
+    ev[1] = e4.y;
+    ev[2] = e4.z;
+    ev[3] = e4.w;
+  } else {
+    load_lane<ACC, VEC, WIN>(prm, w, i0, d, ev);
+  }
+}
+
 // W <= 2: one thread = four consecutive coordinates of every worker in the group.
 //   ACC: accumulate (u, e update) before inserting e; otherwise insert e as given.
 //   VEC: all vectors 16-byte aligned (float4 path for full quads).
@@ -159,6 +187,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_
   const int64_t d = prm.d;
   const int64_t nq = (d + 3) / 4;
   const int64_t qstride = (int64_t)gridDim.x * (blockDim.x / G);
+  const uint64_t pol_stream = policy_evict_first(), pol_table = policy_evict_last();
   for (int64_t q = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / G; q < nq; q += qstride) {
     const int64_t i0 = q * 4;
     float ev[4][4];
@@ -166,7 +195,7 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_
     for (int w4 = 0; w4 < 4; ++w4) {
       const int w = sub * 4 + w4;
       if (w < prm.nw) {
-        load_lane<ACC, VEC, WIN>(prm, w, i0, d, ev[w4]);
+        load_lane_hinted<ACC, VEC, WIN>(prm, w, i0, d, ev[w4], pol_stream);
       } else {
 #pragma unroll
         for (int t = 0; t < 4; ++t) ev[w4][t] = 0.f;
@@ -184,8 +213,8 @@ __global__ void __launch_bounds__(kBlock) k_accumulate_insert_coop(const __grid_
         if (t < tmax) {
           const uint32_t bk = bucket_of<POW2>(x, prm.c, prm.cmask);
           const uint32_t sb = signbit_of(y);
-          red_add_v4(row + (size_t)bk * W, apply_sign(ev[0][t], sb), apply_sign(ev[1][t], sb),
-                     apply_sign(ev[2][t], sb), apply_sign(ev[3][t], sb));
+          red_add_v4_keep(row + (size_t)bk * W, apply_sign(ev[0][t], sb), apply_sign(ev[1][t], sb),
+                          apply_sign(ev[2][t], sb), apply_sign(ev[3][t], sb), pol_table);
           x = step61(x, a);
           y = step61(y, a2);
         }
