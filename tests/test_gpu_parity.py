@@ -786,3 +786,27 @@ def _check_heavymix_against_oracle(H, idx, est, l2sq, est_o, l2_o, band, k, fill
     else:
         masked_o = np.where(h_o, est_o, 0.0)
         H.check_topk_set(idx, oracle.topk(masked_o, k), masked_o, band + slack, k, est_o.size)
+
+
+def _random_step_configs(n, seed=2108):
+    """Seeded draws of small step shapes: P in 1..20, d up to 300,000 (often ragged), r in 1..9,
+    c a power of two or not, k from 1 to d, and every group width the library accepts."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(n):
+        P = int(rng.integers(1, 21))
+        d = int(rng.choice([rng.integers(1, 100), rng.integers(100, 300_001)]))
+        r = int(rng.integers(1, 10))
+        c = int(2 ** rng.integers(0, 16)) if rng.random() < 0.6 else int(rng.integers(1, 40_000))
+        k = int(rng.integers(1, d + 1)) if rng.random() < 0.3 else int(min(d, rng.integers(1, 2000)))
+        W = int(rng.choice([0, 0, 1, 2, 4, 8, 16]))
+        out.append((P, d, r, c, k, W))
+    return out
+
+
+@pytest.mark.parametrize("P,d,r,c,k,W", _random_step_configs(16))
+def test_random_step_shapes(gs, H, P, d, r, c, k, W):
+    """Two steps of randomly drawn shapes against the oracle, with every agreement check of the
+    step tests (tables, merged table, estimate band, selection, state, gathered values)."""
+    w = workloads.get_config("tiny-2^20")
+    _run_steps(gs, H, w, d, 2, c=c, k=k, r=r, P=P, group_width=W, seed=d % 997 + r)
