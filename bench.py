@@ -417,7 +417,7 @@ def launches_per_step(run: Runner, variant: str) -> int:
     prunes = variant != "heavymix" and w.d >= PRUNE_MIN_DIM and w.r >= 3 and (w.c & (w.c - 1)) == 0
     inserts = run.groups * run.passes
     if variant == "heavymix":
-        query = 4 + 6                                 # sumsq, theta, query, keys + selection
+        query = 3 + 6                                 # sumsq, theta, query (with the keys) + selection
     else:
         query = 1 + 6 + (2 if prunes else 0)          # query + selection (+ sample and repair check)
     tail = 6 if variant == "sketched_state" else 1

@@ -3,7 +3,7 @@
 //
 // The selection is a radix select on a 32-bit key in three levels: bits 31..21, 20..10 and
 // 9..0.  For the top-k by |est| the key is the bit pattern of |est| (for non-negative floats
-// it orders like the value); HEAVYMIX selects on a composite key (see k_heavy_keys).  Each
+// it orders like the value); HEAVYMIX selects on a composite key (see heavy_key).  Each
 // histogram kernel ends with a pick: the last CTA to finish (found with a counter after a
 // memory fence, so no CTA waits for another) finds the bin that holds the k-th largest key
 // and how many keys of that bin are still to be taken.  After three levels the k-th largest
@@ -185,6 +185,26 @@ __device__ __forceinline__ float median_of(float (&v)[R]) {
   return 0.5f * (v[R / 2 - 1] + v[R / 2]);
 }
 
+// The i-th output (i = 0, 1, ...) of the splitmix64 stream seeded with `seed`: the state after
+// i + 1 increments of the golden-ratio constant, mixed (Steele, Lea and Flood, 2014).
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t i) {
+  uint64_t z = seed + (i + 1) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Composite key of HEAVYMIX.  Members of H = {i : est_i^2 >= theta} get 0x80000000 | bits(|est_i|):
+// all of H ranks above all of NH, and inside H by |est|.  Members of NH get 0x7FFFFFFF - xi_i,
+// xi_i = the top 31 bits of splitmix64_at(fill_seed, i): the largest NH keys are the NH
+// coordinates with the smallest xi, a uniformly random subset (rand_l(NH)).  The top-k of these
+// keys (ties to the smaller index) is H plus k - |H| random coordinates of NH when |H| < k, and
+// the k largest |est| of H otherwise.
+__device__ __forceinline__ uint32_t heavy_key(float e, double theta, uint64_t fill_seed, uint64_t i) {
+  const double e2 = (double)e * (double)e;  // exact
+  return e2 >= theta ? (0x80000000u | key_of(e)) : 0x7FFFFFFFu - (uint32_t)(splitmix64_at(fill_seed, i) >> 33);
+}
+
 struct QueryParams {
   const float* T;     // merged table [r][c]
   float* est;         // [d]
@@ -197,6 +217,10 @@ struct QueryParams {
   int32_t vec;        // est 16-byte aligned
   int32_t hist_on;    // build the level-1 histogram of |est| keys and pick
   int32_t prune;      // skip rows below st->prune_key (estimate internal to the workspace)
+  uint32_t* keys;     // HEAVYMIX: also store each coordinate's composite key here, and build the
+                      // level-1 histogram (and pick) on those keys instead of |est|
+  const double* theta;  // HEAVYMIX: the threshold l2sq / k of H
+  uint64_t fill_seed;   // HEAVYMIX: the seed of the random fill
   HashCoeffs h;
 };
 
@@ -228,7 +252,8 @@ __device__ __forceinline__ void store_est(const QueryParams& prm, int64_t i0, in
 
 // Fast path: R rows known at compile time, c a power of two.  A thread takes four consecutive
 // coordinates; their hash values after the first come from the incremental form.
-template <int R>
+// HM: HEAVYMIX mode (prm.keys set): each coordinate's composite key is stored and histogrammed.
+template <int R, bool HM = false>
 __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryParams prm) {
   grid_begin();
   __shared__ uint32_t sh[kBins];
@@ -238,12 +263,14 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int lane = threadIdx.x & 31;
   const uint32_t pk = prune_key_of(prm);
+  const double theta = HM ? __ldcg(prm.theta) : 0.0;
   constexpr int kF = R / 2 + 1;  // rows that bound the median
   for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += stride) {
     const int64_t q = q0 + lane;
     const int64_t i0 = q * 4;
     const int tmax = q < nq ? (d - i0 < 4 ? (int)(d - i0) : 4) : 0;
     float m[4] = {0.f, 0.f, 0.f, 0.f};
+    uint32_t hk[4] = {0u, 0u, 0u, 0u};
     if (tmax > 0) {
       float v[4][R];
 #pragma unroll
@@ -287,10 +314,20 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
 #pragma unroll
       for (int t = 0; t < 4; ++t) m[t] = need[t] ? median_of<R>(v[t]) : __uint_as_float(kPrunedBits);
       store_est(prm, i0, tmax, m);
+      if (HM) {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) hk[t] = heavy_key(m[t], theta, prm.fill_seed, (uint64_t)(i0 + t));
+        if (tmax == 4) {
+          *reinterpret_cast<uint4*>(prm.keys + i0) = make_uint4(hk[0], hk[1], hk[2], hk[3]);
+        } else {
+          for (int t = 0; t < tmax; ++t) prm.keys[i0 + t] = hk[t];
+        }
+      }
     }
     if (prm.hist_on) {
 #pragma unroll
-      for (int t = 0; t < 4; ++t) hist_add(sh, t < tmax ? (key_of(m[t]) >> kL1Shift) : kNone);
+      for (int t = 0; t < 4; ++t)
+        hist_add(sh, t < tmax ? ((HM ? hk[t] : key_of(m[t])) >> kL1Shift) : kNone);
     }
   }
   if (prm.hist_on) {
@@ -460,6 +497,7 @@ __global__ void __launch_bounds__(kBlock) k_query_generic(const __grid_constant_
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int lane = threadIdx.x & 31;
   const int r = prm.r;
+  const double theta = prm.keys ? __ldcg(prm.theta) : 0.0;
   for (int64_t i0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < d; i0 += stride) {
     const int64_t i = i0 + lane;
     uint32_t bin = kNone;
@@ -482,7 +520,12 @@ __global__ void __launch_bounds__(kBlock) k_query_generic(const __grid_constant_
       }
       const float m = (r & 1) ? v[r / 2] : 0.5f * (v[r / 2 - 1] + v[r / 2]);
       prm.est[i] = m;
-      bin = key_of(m) >> kL1Shift;
+      uint32_t key = key_of(m);
+      if (prm.keys) {
+        key = heavy_key(m, theta, prm.fill_seed, (uint64_t)i);
+        prm.keys[i] = key;
+      }
+      bin = key >> kL1Shift;
     }
     if (prm.hist_on) hist_add(sh, bin);
   }
@@ -954,49 +997,6 @@ __global__ void k_heavy_theta(const double* __restrict__ sumsq, int r, int64_t k
   }
 }
 
-// The i-th output (i = 0, 1, ...) of the splitmix64 stream seeded with `seed`: the state after
-// i + 1 increments of the golden-ratio constant, mixed (Steele, Lea and Flood, 2014).
-__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t i) {
-  uint64_t z = seed + (i + 1) * 0x9E3779B97F4A7C15ull;
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
-
-// Composite key of HEAVYMIX.  Members of H = {i : est_i^2 >= theta} get 0x80000000 | bits(|est_i|):
-// all of H ranks above all of NH, and inside H by |est|.  Members of NH get 0x7FFFFFFF - xi_i,
-// xi_i = the top 31 bits of splitmix64_at(fill_seed, i): the largest NH keys are the NH
-// coordinates with the smallest xi, a uniformly random subset (rand_l(NH)).  The top-k of these
-// keys (ties to the smaller index) is H plus k - |H| random coordinates of NH when |H| < k, and
-// the k largest |est| of H otherwise.  Ends with the level-1 histogram and pick.
-__global__ void __launch_bounds__(kBlock) k_heavy_keys(const float* __restrict__ est, int64_t d,
-                                                       const double* __restrict__ theta_p, uint64_t fill_seed,
-                                                       uint32_t* __restrict__ keys, uint32_t* hist1, SelectState* st,
-                                                       uint32_t k) {
-  grid_begin();
-  __shared__ uint32_t sh[kBins];
-  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
-  __syncthreads();
-  const double theta = __ldcg(theta_p);
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  const int lane = threadIdx.x & 31;
-  for (int64_t i0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < d; i0 += stride) {
-    const int64_t i = i0 + lane;
-    uint32_t bin = kNone;
-    if (i < d) {
-      const float e = est[i];
-      const double e2 = (double)e * (double)e;  // exact
-      const uint32_t key = e2 >= theta ? (0x80000000u | key_of(e))
-                                       : 0x7FFFFFFFu - (uint32_t)(splitmix64_at(fill_seed, (uint64_t)i) >> 33);
-      keys[i] = key;
-      bin = key >> kL1Shift;
-    }
-    hist_add(sh, bin);
-  }
-  hist_flush(sh, hist1, kBins);
-  last_block_pick(hist1, 11, st, 0, k);
-}
-
 // ---- launchers -----------------------------------------------------------------------------
 
 template <typename K>
@@ -1008,7 +1008,7 @@ int persistent_grid(K kernel, int64_t work_items, int block) {
 
 template <int R>
 cudaError_t launch_query_r(const QueryParams& p, cudaStream_t s) {
-  auto kern = k_query<R>;
+  auto kern = p.keys ? k_query<R, true> : k_query<R, false>;
   launch(kern, persistent_grid(kern, (p.d + 3) / 4, kBlock), kBlock, s, p);
   return cudaGetLastError();
 }
@@ -1116,6 +1116,9 @@ QueryParams make_query_params(const float* merged, const HashCoeffs& h, int r, u
   qp.vec = (reinterpret_cast<uintptr_t>(est) & 15u) == 0 ? 1 : 0;
   qp.hist_on = 1;
   qp.prune = 0;
+  qp.keys = nullptr;
+  qp.theta = nullptr;
+  qp.fill_seed = 0;
   qp.h = h;
   return qp;
 }
@@ -1261,12 +1264,13 @@ cudaError_t launch_query_heavymix(const float* merged, const HashCoeffs& h, int 
   launch(k_row_sumsq, dim3(gx, r), kBlock, s, merged, c, sumsq);
   const int prune = (!est_out && can_prune(r, c, d)) ? 1 : 0;
   launch(k_heavy_theta, 1, 32, s, sumsq, r, k, theta, l2sq_out, w.st, prune);
+  // the query stores each coordinate's composite key and picks on their level-1 histogram
   QueryParams qp = make_query_params(merged, h, r, c, d, k, est, w.hist, w.st);
-  qp.hist_on = 0;
   qp.prune = prune;
+  qp.keys = keys;
+  qp.theta = theta;
+  qp.fill_seed = fill_seed;
   if ((err = launch_query(qp, s)) != cudaSuccess) return err;
-  launch(k_heavy_keys, persistent_grid(k_heavy_keys, d, kBlock), kBlock, s, est, d, theta, fill_seed, keys, w.hist,
-                                                                           w.st, (uint32_t)k);
   if ((err = mark(marks, 1, s)) != cudaSuccess) return err;
   if ((err = select_from_keys(w, reinterpret_cast<const float*>(keys), 1, 0xFFFFFFFFu, d, k, idx_out, s)) !=
       cudaSuccess)
