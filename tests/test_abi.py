@@ -102,3 +102,32 @@ def test_no_cpu_fallback_when_library_missing(tmp_path, monkeypatch):
     monkeypatch.setattr(gs, "LIB_PATH", str(tmp_path / "absent.so"))
     with pytest.raises(ImportError):
         gs.gs_sketch_create(5, 16, 1, 4)
+
+
+def test_validation_of_the_later_entry_points(lib):
+    """The entry points added for merging separate sketches, the HEAVYMIX step, the staged
+    insert, the measurement aids and the plan query timings reject bad arguments on the host."""
+    import paper_2108_06004_gb300 as gs
+    arr = (ctypes.c_void_p * 2)(16, 32)
+    assert lib.gs_sketch_merge_sketches(None, 1, None) == gs.GS_ERR_INVALID_ARG
+    none2 = (ctypes.c_void_p * 2)(None, None)
+    assert lib.gs_sketch_merge_sketches(none2, 0, None) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_sketch_merge_sketches(none2, 65, None) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_sketch_merge_sketches(none2, 2, None) == gs.GS_ERR_INVALID_ARG   # NULL sketch
+    sz = ctypes.c_size_t()
+    assert lib.gs_heavymix_step_workspace_size(0, 1, ctypes.byref(sz)) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_heavymix_step_workspace_size(1000, 10, ctypes.byref(sz)) == gs.GS_OK and sz.value >= 8000
+    assert lib.gs_heavymix_step(None, arr, arr, arr, 10, 0.9, 1, 7, 64, 128, None, 256, 1 << 20, None) \
+        == gs.GS_ERR_INVALID_ARG
+    plan = ctypes.c_void_p(1)
+    assert lib.gs_heavymix_step_plan_create(None, arr, arr, arr, 10, 0.9, 1, 7, 64, 128, None, 256, 1 << 20, 0,
+                                            ctypes.byref(plan)) == gs.GS_ERR_INVALID_ARG
+    assert plan.value is None
+    assert lib.gs_accumulate_insert_staged(None, 0, 1, arr, arr, arr, 10, 0.9, None) == gs.GS_ERR_INVALID_ARG
+    ms = ctypes.c_float()
+    assert lib.gs_insert_request_ceiling(None, 10, 256, 1 << 20, ctypes.byref(ms), None) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_insert_request_ceiling_window_size(None, ctypes.byref(sz)) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_query_request_ceiling(None, 10, 256, 1 << 20, ctypes.byref(ms), None) == gs.GS_ERR_INVALID_ARG
+    n_out = ctypes.c_int32()
+    assert lib.gs_plan_query_times(None, None, None, 1, ctypes.byref(n_out)) == gs.GS_ERR_INVALID_ARG
+    assert lib.gs_query_topk_noalloc(None, 10, 1, 64, 128, None) == gs.GS_ERR_INVALID_ARG
