@@ -38,13 +38,25 @@ namespace {
 
 thread_local std::string g_err;
 
-gs_status fail(gs_status st, const std::string& msg) {
-  g_err = msg;
+// Record the message of a failing call; a message that cannot be stored is dropped, so that
+// the status still reaches the caller.
+gs_status fail(gs_status st, const char* msg) noexcept {
+  try {
+    g_err = msg;
+  } catch (...) {
+    g_err.clear();
+  }
   return st;
 }
 
-gs_status cuda_fail(cudaError_t e, const char* what) {
-  g_err = std::string(what) + ": " + cudaGetErrorString(e);
+gs_status fail(gs_status st, const std::string& msg) noexcept { return fail(st, msg.c_str()); }
+
+gs_status cuda_fail(cudaError_t e, const char* what) noexcept {
+  try {
+    g_err = std::string(what) + ": " + cudaGetErrorString(e);
+  } catch (...) {
+    g_err.clear();
+  }
   return GS_ERR_CUDA;
 }
 
@@ -639,6 +651,7 @@ gs_status gs_sketch_create(int32_t r, int32_t c, uint64_t seed, int32_t workers,
 }
 
 gs_status gs_sketch_destroy(gs_sketch* sk) {
+  GS_GUARD_BEGIN
   if (!sk) return GS_OK;
   int prev = -1;
   cudaGetDevice(&prev);
@@ -648,10 +661,12 @@ gs_status gs_sketch_destroy(gs_sketch* sk) {
   delete sk;
   if (e != cudaSuccess) return cuda_fail(e, "cudaFree");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_info(const gs_sketch* sk, int32_t* r, int32_t* c, int32_t* workers, int32_t* group_width,
                          int32_t* rows_per_pass) {
+  GS_GUARD_BEGIN
   if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
   if (r) *r = sk->r;
   if (c) *c = sk->c;
@@ -659,9 +674,11 @@ gs_status gs_sketch_info(const gs_sketch* sk, int32_t* r, int32_t* c, int32_t* w
   if (group_width) *group_width = sk->W;
   if (rows_per_pass) *rows_per_pass = sk->rows_per_pass;
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_coefficients(const gs_sketch* sk, uint64_t* out4r) {
+  GS_GUARD_BEGIN
   if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
   if (!out4r) return fail(GS_ERR_INVALID_ARG, "out4r is NULL");
   for (int j = 0; j < sk->r; ++j) {
@@ -671,17 +688,21 @@ gs_status gs_sketch_coefficients(const gs_sketch* sk, uint64_t* out4r) {
     out4r[4 * j + 3] = sk->h.b2[j];
   }
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_zero(gs_sketch* sk, gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   const size_t bytes = ((size_t)sk->groups * sk->r * sk->c * sk->W + (size_t)sk->r * sk->c) * sizeof(float);
   cudaError_t e = cudaMemsetAsync(sk->tables, 0, bytes, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_accumulate(float* momentum, float* error, const float* grad, int64_t d, float rho, gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_vec(momentum, "momentum"));
   GS_TRY(check_vec(error, "error"));
   GS_TRY(check_vec(grad, "grad"));
@@ -689,9 +710,11 @@ gs_status gs_accumulate(float* momentum, float* error, const float* grad, int64_
   cudaError_t e = gs::launch_accumulate(momentum, error, grad, d, rho, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "accumulate launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_insert(gs_sketch* sk, int32_t worker, const float* vec, int64_t d, gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   GS_TRY(check_vec(vec, "vec"));
   GS_TRY(check_d(d));
@@ -713,6 +736,7 @@ gs_status gs_sketch_insert(gs_sketch* sk, int32_t worker, const float* vec, int6
   cudaError_t e = gs::launch_insert_lane(p, W, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "insert launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_accumulate_insert(gs_sketch* sk, int32_t first_worker, int32_t n_workers, float* const* momentum,
@@ -779,6 +803,7 @@ gs_status gs_accumulate_insert_staged(gs_sketch* sk, int32_t first_worker, int32
 }
 
 gs_status gs_sketch_merge_tree(gs_sketch* sk, int32_t P, gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   if (P < 1 || P > sk->workers) return fail(GS_ERR_INVALID_ARG, "P must lie in [1, workers]");
   gs::MergeParams mp;
@@ -790,6 +815,7 @@ gs_status gs_sketch_merge_tree(gs_sketch* sk, int32_t P, gs_stream stream) {
   cudaError_t e = gs::launch_merge(mp, sk->W, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "merge launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_merge_sketches(gs_sketch* const* sketches, int32_t P, gs_stream stream) {
@@ -819,15 +845,18 @@ gs_status gs_sketch_merge_sketches(gs_sketch* const* sketches, int32_t P, gs_str
 }
 
 gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_GUARD_BEGIN
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
   if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
   *bytes = gs::query_topk_workspace_bytes(d, k);
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_out, float* est_out,
                         void* workspace, size_t workspace_bytes, gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
@@ -840,19 +869,23 @@ gs_status gs_query_topk(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_
                                         as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "query/top-k launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_query_heavymix_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_GUARD_BEGIN
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
   if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
   *bytes = gs::heavymix_workspace_bytes(d, k);
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_query_heavymix(const gs_sketch* sk, int64_t d, int64_t k, uint64_t fill_seed, int64_t* idx_out,
                             float* est_out, double* l2sq_out, void* workspace, size_t workspace_bytes,
                             gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
@@ -866,6 +899,7 @@ gs_status gs_query_heavymix(const gs_sketch* sk, int64_t d, int64_t k, uint64_t 
                                             est_out, l2sq_out, workspace, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "HEAVYMIX launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_query_topk_noalloc(const gs_sketch* sk, int64_t d, int64_t k, int64_t* idx_out, float* est_out,
@@ -947,6 +981,7 @@ gs_status gs_gather_zero_update(float* const* momentum, float* const* error, int
 
 gs_status gs_apply_update(float* weights, int64_t d, const int64_t* idx, const float* vals, int64_t k, float lr,
                           gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_vec(weights, "weights"));
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
@@ -955,14 +990,17 @@ gs_status gs_apply_update(float* weights, int64_t d, const int64_t* idx, const f
   cudaError_t e = gs::launch_apply_update(weights, d, idx, vals, k, lr, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "update launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_step_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_GUARD_BEGIN
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
   if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
   *bytes = step_ws_bytes(d, k);
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_step(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad, int64_t d,
@@ -986,11 +1024,13 @@ gs_status gs_train_step(gs_sketch* sk, float* weights, float lr, float* const* m
 }
 
 gs_status gs_heavymix_step_workspace_size(int64_t d, int64_t k, size_t* bytes) {
+  GS_GUARD_BEGIN
   GS_TRY(check_d(d));
   if (k < 1 || k > d) return fail(GS_ERR_INVALID_ARG, "k must lie in [1, d]");
   if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
   *bytes = gs::heavymix_workspace_bytes(d, k);
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_heavymix_step(gs_sketch* sk, float* const* momentum, float* const* error, const float* const* grad,
@@ -1011,13 +1051,16 @@ gs_status gs_heavymix_step(gs_sketch* sk, float* const* momentum, float* const* 
 }
 
 gs_status gs_sketch_merged_table(const gs_sketch* sk, float** table_out) {
+  GS_GUARD_BEGIN
   if (!sk) return fail(GS_ERR_INVALID_ARG, "sketch is NULL");
   if (!table_out) return fail(GS_ERR_INVALID_ARG, "table_out is NULL");
   *table_out = sk->merged;
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_query_at(const gs_sketch* sk, const int64_t* idx, int64_t k, float* est_out, gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   if (k < 1) return fail(GS_ERR_INVALID_ARG, "k must be positive");
   if (!idx || !aligned(idx, 8)) return fail(GS_ERR_INVALID_ARG, "idx is NULL or not 8-byte aligned");
@@ -1025,10 +1068,12 @@ gs_status gs_sketch_query_at(const gs_sketch* sk, const int64_t* idx, int64_t k,
   cudaError_t e = gs::launch_query_at(sk->merged, sk->h, sk->r, (uint32_t)sk->c, idx, k, est_out, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "query_at launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_add_sparse(gs_sketch* sk, const int64_t* idx, const float* vals, int64_t k, float scale,
                                gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   if (k < 1) return fail(GS_ERR_INVALID_ARG, "k must be positive");
   if (!idx || !aligned(idx, 8)) return fail(GS_ERR_INVALID_ARG, "idx is NULL or not 8-byte aligned");
@@ -1037,6 +1082,7 @@ gs_status gs_sketch_add_sparse(gs_sketch* sk, const int64_t* idx, const float* v
                                         as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "add_sparse launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketched_state_step(gs_sketch* workers, gs_sketch* momentum, gs_sketch* error, const float* const* grad,
@@ -1137,6 +1183,7 @@ gs_status gs_sketched_state_plan_create(gs_sketch* workers, gs_sketch* momentum,
 }
 
 gs_status gs_plan_launch(gs_plan* plan, gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_plan(plan));
   cudaError_t e = cudaSuccess;
   const size_t slot = (size_t)(plan->launches % kPlanRing);
@@ -1147,6 +1194,7 @@ gs_status gs_plan_launch(gs_plan* plan, gs_stream stream) {
   if (e != cudaSuccess) return cuda_fail(e, "cudaGraphLaunch");
   ++plan->launches;
   return GS_OK;
+  GS_GUARD_END
 }
 
 }  // extern "C"
@@ -1175,13 +1223,16 @@ gs_status plan_mark_times(gs_plan* plan, int a, int b, float* ms_out, int32_t n,
 extern "C" {
 
 gs_status gs_plan_insert_times(gs_plan* plan, float* ms_out, int32_t n, int32_t* n_out) {
+  GS_GUARD_BEGIN
   GS_TRY(check_plan(plan));
   if (!(plan->flags & GS_PLAN_TIME_INSERT)) return fail(GS_ERR_INVALID_ARG, "the plan was created without GS_PLAN_TIME_INSERT");
   if (!ms_out || !n_out || n < 0) return fail(GS_ERR_INVALID_ARG, "ms_out or n_out is NULL, or n < 0");
   return plan_mark_times(plan, kInsertBegin, kInsertEnd, ms_out, n, n_out);
+  GS_GUARD_END
 }
 
 gs_status gs_plan_query_times(gs_plan* plan, float* query_ms_out, float* select_ms_out, int32_t n, int32_t* n_out) {
+  GS_GUARD_BEGIN
   GS_TRY(check_plan(plan));
   if (!(plan->flags & GS_PLAN_TIME_QUERY)) return fail(GS_ERR_INVALID_ARG, "the plan was created without GS_PLAN_TIME_QUERY");
   if (!query_ms_out || !select_ms_out || !n_out || n < 0)
@@ -1190,22 +1241,27 @@ gs_status gs_plan_query_times(gs_plan* plan, float* query_ms_out, float* select_
   GS_TRY(plan_mark_times(plan, kQueryBegin, kQueryEnd, query_ms_out, n, n_out));
   GS_TRY(plan_mark_times(plan, kQueryEnd, kSelectEnd, select_ms_out, n, &n2));
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_plan_destroy(gs_plan* plan) {
+  GS_GUARD_BEGIN
   if (!plan) return GS_OK;
   cudaError_t e = cudaSuccess;
   if (plan->launches > 0) e = cudaDeviceSynchronize();
   plan_free(plan);
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_insert_request_ceiling_window_size(const gs_sketch* sk, size_t* bytes) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   if (!bytes) return fail(GS_ERR_INVALID_ARG, "bytes is NULL");
   *bytes = (size_t)3 * sk->W * GS_CEILING_WINDOW_FLOATS * sizeof(float);
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_insert_request_ceiling(gs_sketch* sk, int64_t d, void* window, size_t window_bytes, float* ms_out,
@@ -1294,6 +1350,7 @@ gs_status gs_query_request_ceiling(const gs_sketch* sk, int64_t d, void* window,
 
 gs_status gs_hash_eval(const gs_sketch* sk, const int64_t* coords, int64_t n, int32_t* bucket_out, int8_t* sign_out,
                        gs_stream stream) {
+  GS_GUARD_BEGIN
   GS_TRY(check_sketch(sk));
   if (n < 1) return fail(GS_ERR_INVALID_ARG, "n must be positive");
   if (!coords || !aligned(coords, 8)) return fail(GS_ERR_INVALID_ARG, "coords is NULL or not 8-byte aligned");
@@ -1301,6 +1358,7 @@ gs_status gs_hash_eval(const gs_sketch* sk, const int64_t* coords, int64_t n, in
   cudaError_t e = gs::launch_hash_eval(sk->h, sk->r, (uint32_t)sk->c, coords, n, bucket_out, sign_out, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail(e, "hash_eval launch");
   return GS_OK;
+  GS_GUARD_END
 }
 
 gs_status gs_sketch_copy_to_host(const gs_sketch* sk, int32_t worker, float* host_out) {
