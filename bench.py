@@ -393,12 +393,16 @@ class Runner:
         return {"insert": mean(ins), "query": None, "select": None, "query_select": mean(per_step("query")),
                 "gen": mean(per_step("gen")), "n": len(ins)}
 
-    def pruned_fraction(self):
-        """Fraction of coordinates whose last query stopped after r/2 + 1 rows (stored -0.0)."""
+    def query_rows(self):
+        """(fraction of coordinates that stopped early, rows read per coordinate) in the last
+        query: a coordinate that stopped after n rows leaves -(n * 2^-149) as its estimate."""
         import torch
-        d = self.w.d
-        est = self.ws[: 4 * d].view(torch.int32)
-        return float((est == -2**31).sum().item()) / d
+        d, r = self.w.d, self.w.r
+        bits = self.ws[: 4 * d].view(torch.int32)
+        marked = (bits > -2**31) & (bits <= -2**31 + 16)
+        n_marked = int(marked.sum().item())
+        rows_marked = int((bits[marked].to(torch.int64) + 2**31).sum().item())
+        return n_marked / d, (rows_marked + (d - n_marked) * r) / d
 
     def close(self):
         for plan in self.plans:
@@ -469,7 +473,8 @@ def time_steps(run: Runner, steps: int, warmup: int, world: int, dev, sampler=No
     return elapsed, n_warm, n_by_plan
 
 
-def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dict, pruned: float):
+def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dict, pruned: float,
+              rows_read: float):
     """The insert-phase roofline (HBM, with the measured request ceiling as co-bound) and the
     median query's (L1->L2 requests against the measured gather ceiling; HBM bytes alongside)."""
     w = run.w
@@ -517,17 +522,16 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
     q = None
     q_ms = ph["query"]
     if q_ms is not None and variant != "heavymix":
-        kf = r // 2 + 1
         prunes = d >= PRUNE_MIN_DIM and r >= 3 and (w.c & (w.c - 1)) == 0
         nq = (d + 3) // 4
         n_s = 4 * ((nq + SAMPLE_PERIOD // 4 - 1) // (SAMPLE_PERIOD // 4)) if prunes else 0
-        requests = d * kf + d * (r - kf) * (1.0 - pruned) + n_s * r
+        requests = d * rows_read + n_s * r
         g_ms = probes.get("query_ms")
         ach = requests / (q_ms / 1e3) / 1e9
         q = {
             "kernel": f"k_qsample + k_query<{r}> + k_repair (median query, S4)" if prunes else f"k_query<{r}> (S4)",
             "bound": "L1->L2 requests (scattered 4-byte reads of the merged table)",
-            "avg_ms": round(q_ms, 4), "pruned_fraction": round(pruned, 4),
+            "avg_ms": round(q_ms, 4), "pruned_fraction": round(pruned, 4), "rows_read_per_coord": round(rows_read, 3),
             "requests_per_step": requests, "requests_per_coord": round(requests / d, 3),
             "achieved_G_requests_per_s": round(ach, 1),
             "peak_G_requests_per_s": None if g_ms is None else round(d * r / (g_ms / 1e3) / 1e9, 1),
@@ -572,9 +576,9 @@ def measure(gs, w, variant, eager, steps, warmup, world, rank, dev, stream, peak
     torch.cuda.synchronize()
     elapsed_ms, n_warm, n_by_plan = time_steps(run, steps, warmup, world, dev, sampler, flush)
     ph = run.phase_times(n_by_plan)
-    pruned = run.pruned_fraction() if variant != "heavymix" else 0.0
+    pruned, rows_read = run.query_rows() if variant != "heavymix" else (0.0, float(run.w.r))
     pr = probe_ceilings(run) if probes else {}
-    k1, q = rooflines(run, variant, ph, peaks, peak_kind, pr, pruned)
+    k1, q = rooflines(run, variant, ph, peaks, peak_kind, pr, pruned, rows_read)
     value = whole_job_rate(world, w.P, w.d, steps, elapsed_ms / 1e3)
     res = {
         "value": value, "ms_per_step": round(elapsed_ms / steps, 4), "steps": steps, "warmup_steps_run": n_warm,
@@ -653,6 +657,7 @@ def short_summary(res: dict, w) -> dict:
                    "request_ceiling_ms": k1["co_bound"]["peak_ms"], "frac_of_request_ceiling": k1["co_bound"]["frac"],
                    "request_ceiling_frac_of_hbm": k1["co_bound"]["peak_frac_of_hbm"]},
         "query": None if q is None else {"avg_ms": q["avg_ms"], "pruned_fraction": q["pruned_fraction"],
+                                          "rows_read_per_coord": q["rows_read_per_coord"],
                                           "achieved_G_requests_per_s": q["achieved_G_requests_per_s"],
                                           "peak_G_requests_per_s": q["peak_G_requests_per_s"], "frac": q["frac"],
                                           "select_ms": q["select_ms"]},

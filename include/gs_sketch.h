@@ -169,9 +169,11 @@ gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * workspace must hold gs_query_topk_workspace_size(d, k) bytes, 256-byte aligned (about
  * 12.3 bytes per coordinate: the estimate, room for a candidate list of (index, key) pairs,
  * and two d-bit bitmaps).
- * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, the query may skip rows: a
- * coordinate whose first r/2 + 1 cells are all below a threshold cannot be selected (they
- * bound the median), and its estimate is left at -0.0 in the workspace.  The threshold is
+ * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, the query may skip rows.  Rows
+ * are read in order, and a coordinate stops once, with f = r/2 + 1, at least f of the cells
+ * read are below a threshold t and at least f are above -t: then |est| < t whatever the
+ * other rows hold, and it cannot be selected.  Its estimate is left in the workspace as
+ * -(n * 2^-149), n the rows it read (f <= n < r).  The threshold is
  * taken by the same call before the main pass, from the full estimate of a fixed sample (the
  * first four coordinates of every 256): the level-1 bin edge below a rank of the sample chosen
  * so that the threshold lies under the k-th largest |est| except with negligible probability.
@@ -195,10 +197,11 @@ gs_status gs_query_heavymix_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * i counted from 0, ties to the smaller index.  idx_out (int64[k]) is ascending; est_out
  * (fp32[d]) and l2sq_out (one device double) may be NULL.  workspace must hold
  * gs_query_heavymix_workspace_size(d, k) bytes, 256-byte aligned.
- * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, a coordinate whose first
- * r/2 + 1 cells all lie below sqrt(l2sq / k) skips its other rows (its est^2 is below the
- * threshold, so it can only enter through the fill) and its estimate is left at -0.0 in the
- * workspace; idx_out is the same as without skipping. */
+ * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, rows are skipped as in
+ * gs_query_topk with t = sqrt(l2sq / k) (rounded down to a bin edge): a coordinate that stops
+ * has est^2 below the threshold, so it can only enter through the fill, and its estimate is
+ * left in the workspace as -(n * 2^-149), n the rows it read; idx_out is the same as without
+ * skipping. */
 gs_status gs_query_heavymix(const gs_sketch* sketch, int64_t d, int64_t k, uint64_t fill_seed,
                             int64_t* idx_out, float* est_out, double* l2sq_out, void* workspace,
                             size_t workspace_bytes, gs_stream stream);

@@ -15,10 +15,10 @@
 //                 coordinates, its level-1 histogram, and a prune key from it: a lower bound
 //                 on the k-th largest |est| of this query, rounded down to a bin edge
 //   k_query       est_i for every i (fp32) + level-1 histogram + pick; when the estimate stays
-//                 in the workspace, a coordinate whose first r/2 + 1 rows all lie below the
-//                 prune key skips its other rows and stores -0.0 (see below)
+//                 in the workspace, a coordinate whose rows read so far bound its |est| below
+//                 the prune key skips its other rows and stores a marker (see below)
 //   k_repair      runs only if the level-1 pick fell below the prune key: recomputes every
-//                 -0.0 estimate in full, rebuilds the level-1 histogram and picks again
+//                 marked estimate in full, rebuilds the level-1 histogram and picks again
 //   k_cand        one pass over est: keys above the picked level-1 bin are selected for
 //                 certain and set their bit in a d-bit bitmap; keys inside the bin become
 //                 candidates (index, key) and feed the level-2 histogram + pick
@@ -224,16 +224,35 @@ struct QueryParams {
   HashCoeffs h;
 };
 
-// Row pruning.  The median of r values lies between the least and the largest of any
-// r/2 + 1 of them (for even r both middle values do, and so does their fp32 mean).  So a
-// coordinate whose first r/2 + 1 signed cells all have |v| < t has |est| < t and cannot be
-// among the top k when t is at most the k-th largest |est|.  The prune key t is computed by
-// this query itself before k_query runs (k_qsample: from the full estimate of a strided
-// sample of coordinates; HEAVYMIX: from its threshold) and kept in the query's own selection
-// state, so every CTA of k_query and k_repair reads the same value.  It is a level-1 bin
-// edge: whether it was safe is then exactly whether the level-1 pick lands in its bin or
-// above, which k_repair checks.
-constexpr uint32_t kPrunedBits = 0x80000000u;  // -0.0f: the stored estimate of a pruned coordinate
+// Row pruning.  With f = r/2 + 1: if at least f of a coordinate's r signed cells are < t and
+// at least f are > -t, then -t < est < t.  For odd r the median is the f-th smallest and the
+// f-th largest value; for even r the two middle values are the f-th smallest and the f-th
+// largest, and the fp32 mean of two values in (-t, t) stays inside (rounding is monotone and
+// twice an fp32 value is exact).  So a coordinate can stop reading rows as soon as both counts
+// reach f: its |est| < t, and it cannot be among the top k when t is at most the k-th largest
+// |est|.  Rows are read in order; the first f always, each later one only while the coordinate
+// is undecided.  A cell with |v| < t counts on both sides, so f of those settle it after the
+// first f rows; one cell outside (-t, t) among them costs one more row, not all of them.
+// The prune key t is computed by this query itself before k_query runs (k_qsample: from the
+// full estimate of a strided sample of coordinates; HEAVYMIX: from its threshold) and kept in
+// the query's own selection state, so every CTA of k_query and k_repair reads the same value.
+// It is a level-1 bin edge: whether it was safe is then exactly whether the level-1 pick
+// lands in its bin or above, which k_repair checks.
+// A coordinate that stopped early stores -(n * 2^-149), n = the rows it read (f <= n < r):
+// a key in level-1 bin 0 that k_repair recognises and the measurement can count.
+constexpr uint32_t kPrunedBits = 0x80000000u;  // sign bit; the low bits hold the rows read
+
+__device__ __forceinline__ bool is_pruned(uint32_t bits) { return bits - (kPrunedBits + 1u) < (uint32_t)GS_MAX_ROWS; }
+
+// Counts of a coordinate's cells below t (lt) and above -t (gt), on keys: |v| < t is
+// key_of(v) < pk; a NaN counts on neither side.
+__device__ __forceinline__ void tally(float v, uint32_t pk, int& lt, int& gt) {
+  const uint32_t b = __float_as_uint(v), key = b & 0x7FFFFFFFu;
+  const bool inside = key < pk;
+  const bool number = key <= 0x7F800000u;
+  lt += (inside || (number && (b >> 31))) ? 1 : 0;
+  gt += (inside || (number && !(b >> 31))) ? 1 : 0;
+}
 
 __device__ __forceinline__ uint32_t prune_key_of(const QueryParams& prm) {
   return prm.prune ? __ldcg(&prm.st->prune_key) : 0u;
@@ -253,8 +272,9 @@ __device__ __forceinline__ void store_est(const QueryParams& prm, int64_t i0, in
 // Fast path: R rows known at compile time, c a power of two.  A thread takes four consecutive
 // coordinates; their hash values after the first come from the incremental form.
 // HM: HEAVYMIX mode (prm.keys set): each coordinate's composite key is stored and histogrammed.
+// Up to 7 rows the register budget keeps four CTAs per SM (no spills at 64 registers).
 template <int R, bool HM = false>
-__global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryParams prm) {
+__global__ void __launch_bounds__(kBlock, R <= 7 ? 4 : 1) k_query(const __grid_constant__ QueryParams prm) {
   grid_begin();
   __shared__ uint32_t sh[kBins];
   for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
@@ -288,13 +308,17 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
           }
         }
       }
-      bool need[4];
+      // the later rows, each only while the coordinate is undecided
+      int lt[4], gt[4], rows[4];
+      bool done[4];
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
-        bool below = pk != 0u;
+        lt[t] = 0;
+        gt[t] = 0;
 #pragma unroll
-        for (int j = 0; j < kF; ++j) below = below && key_of(v[t][j]) < pk;
-        need[t] = !below;
+        for (int j = 0; j < kF; ++j) tally(v[t][j], pk, lt[t], gt[t]);
+        rows[t] = kF;
+        done[t] = pk != 0u && lt[t] >= kF && gt[t] >= kF;
       }
 #pragma unroll
       for (int j = kF; j < R; ++j) {
@@ -305,18 +329,28 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
         for (int t = 0; t < 4; ++t) {
           v[t][j] = 0.f;
           if (t < tmax) {
-            if (need[t]) v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
+            if (!done[t]) {
+              v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
+              tally(v[t][j], pk, lt[t], gt[t]);
+              ++rows[t];
+            }
             x = step61(x, prm.h.a[j]);
             y = step61(y, prm.h.a2[j]);
           }
         }
+        if (j + 1 < R) {
+#pragma unroll
+          for (int t = 0; t < 4; ++t) done[t] = done[t] || (pk != 0u && lt[t] >= kF && gt[t] >= kF);
+        }
       }
 #pragma unroll
-      for (int t = 0; t < 4; ++t) m[t] = need[t] ? median_of<R>(v[t]) : __uint_as_float(kPrunedBits);
+      for (int t = 0; t < 4; ++t)
+        m[t] = done[t] ? __uint_as_float(kPrunedBits | (uint32_t)rows[t]) : median_of<R>(v[t]);
       store_est(prm, i0, tmax, m);
       if (HM) {
 #pragma unroll
-        for (int t = 0; t < 4; ++t) hk[t] = heavy_key(m[t], theta, prm.fill_seed, (uint64_t)(i0 + t));
+        for (int t = 0; t < 4; ++t)
+          hk[t] = heavy_key(done[t] ? 0.f : m[t], theta, prm.fill_seed, (uint64_t)(i0 + t));
         if (tmax == 4) {
           *reinterpret_cast<uint4*>(prm.keys + i0) = make_uint4(hk[0], hk[1], hk[2], hk[3]);
         } else {
@@ -338,9 +372,10 @@ __global__ void __launch_bounds__(kBlock) k_query(const __grid_constant__ QueryP
 
 // Runs after k_query.  If the level-1 pick landed in the prune key's bin or above, the k-th
 // largest |est| is at least the prune key and pruning changed nothing the selection sees: the
-// kernel returns at once.  Otherwise every stored -0.0 (each pruned coordinate, and any
-// genuine -0.0, which recomputes to itself) gets its full median, the level-1 histogram is
-// rebuilt from all estimates into hist_r, and the level-1 pick is made again.
+// kernel returns at once.  Otherwise every stored marker (each pruned coordinate, and any
+// genuine estimate with the same bits, which recomputes to itself) gets its full median, the
+// level-1 histogram is rebuilt from all estimates into hist_r, and the level-1 pick is made
+// again.
 template <int R>
 __global__ void __launch_bounds__(kBlock) k_repair(const __grid_constant__ QueryParams prm, uint32_t* hist_r) {
   grid_begin();
@@ -357,7 +392,7 @@ __global__ void __launch_bounds__(kBlock) k_repair(const __grid_constant__ Query
     uint32_t bin = kNone;
     if (i < d) {
       float e = prm.est[i];
-      if (__float_as_uint(e) == kPrunedBits) {
+      if (is_pruned(__float_as_uint(e))) {
         float v[R];
 #pragma unroll
         for (int j = 0; j < R; ++j) {

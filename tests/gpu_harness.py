@@ -67,6 +67,16 @@ def host(t: torch.Tensor) -> np.ndarray:
     return t.detach().cpu().numpy()
 
 
+def pruned_rows(e_int: np.ndarray, r: int):
+    """(mask, rows): the coordinates whose workspace estimate is a pruning marker, -(n * 2^-149)
+    with n the rows read, and n for each of them.  Every marker must name r/2 + 1 <= n < r."""
+    bits = e_int.view(np.uint32)
+    mask = (bits > np.uint32(0x80000000)) & (bits <= np.uint32(0x80000010))
+    n = (bits[mask] & np.uint32(0xFF)).astype(np.int64)
+    assert np.all((n >= r // 2 + 1) & (n < r)), "a marker names an impossible row count"
+    return mask, n
+
+
 def worker_tables(run: GpuRun, P: int, r: int, c: int):
     out = []
     for p in range(P):

@@ -185,7 +185,7 @@ def run_full_size(gs, H, name, steps):
                 clock.lap("oracle query")
                 err = np.abs(est_g.astype(np.float64) - est_o)
                 assert np.all(err <= band), f"step {t}: estimate outside its band at {np.nonzero(err > band)[0][:10]}"
-                pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
+                pruned, _ = H.pruned_rows(e_int, r)
                 tau_g = np.abs(est_g[gi]).min()
                 assert np.all(np.abs(est_o[pruned]) <= tau_g + band[pruned]), f"step {t}: a skipped row mattered"
                 idx_o = oracle.topk_by_threshold(est_o, k)

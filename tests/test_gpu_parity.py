@@ -357,10 +357,10 @@ def _prune_input(rng, d, k, adversarial):
     return x
 
 
-def _check_pruned_against_full(H, got, e_int, want, e, k):
+def _check_pruned_against_full(H, got, e_int, want, e, k, r):
     assert np.array_equal(got, want), "selections differ"
     H.check_selection_exact(got, e, k)
-    pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
+    pruned, _ = H.pruned_rows(e_int, r)
     exact = e_int.view(np.uint32) == e.view(np.uint32)
     assert np.all(pruned | exact)
     tau = np.sort(np.abs(e))[-k]
@@ -376,7 +376,8 @@ def test_pruned_query_matches_full_query(gs, H, r, adversarial):
     coordinates stop after r/2 + 1 rows; on adversarial input (every heavy coordinate on the
     sample) the key lies above the k-th largest |est|, and the repair pass must restore every
     skipped estimate.  Either way the selection equals the full query's exactly, every selected
-    estimate is exact, and every skipped (-0.0) one lies below the k-th largest |est|."""
+    estimate is exact, and every skipped one (a marker naming the rows it read) lies below the
+    k-th largest |est|."""
     d, c, k, seed = 4_200_007, 1 << 16, 4000, 40 + r      # pruning applies from d = 2^22
     rng = np.random.default_rng(seed)
     sk = gs.gs_sketch_create(r, c, seed, 1, 0)
@@ -396,7 +397,7 @@ def test_pruned_query_matches_full_query(gs, H, r, adversarial):
             got, e_int = H.host(idx).copy(), H.host(est_int).copy()
             gs.gs_query_topk(sk, d, k, idx_full, est_full, ws)  # caller's estimate: every row
             torch.cuda.synchronize()
-            pruned = _check_pruned_against_full(H, got, e_int, H.host(idx_full), H.host(est_full), k)
+            pruned = _check_pruned_against_full(H, got, e_int, H.host(idx_full), H.host(est_full), k, r)
             if adversarial:
                 assert not pruned.any(), "the repair left skipped estimates"
             else:
@@ -438,6 +439,58 @@ def test_pruned_queries_on_two_streams(gs, H):
     finally:
         for sk in sks:
             gs.gs_sketch_destroy(sk)
+
+
+def _settle_threshold(v, f):
+    """Per column of v (rows x coordinates, the signed cells in the order the query reads them):
+    the least t0 such that every t > t0 has at least f values < t and at least f values > -t,
+    i.e. the larger of the f-th smallest value and minus the f-th largest."""
+    srt = np.sort(v, axis=0)
+    return np.maximum(srt[f - 1], -srt[v.shape[0] - f])
+
+
+@pytest.mark.parametrize("r", [4, 5, 7])
+def test_pruned_rows_follow_the_rule(gs, H, r):
+    """The rows each coordinate read, from its marker, against the rule, with the signed cells
+    recomputed on the host from the merged table and the hash values: one prune key t must
+    exist such that every coordinate that stopped after n rows was settled by its first n cells
+    (t above their settle threshold) and unsettled by its first n - 1 when n > r/2 + 1, and
+    every coordinate that read all r rows was unsettled by its first r - 1."""
+    d, c, k, seed = 4_200_007, 1 << 16, 4000, 60 + r
+    f = r // 2 + 1
+    rng = np.random.default_rng(seed)
+    sk = gs.gs_sketch_create(r, c, seed, 1, 0)
+    try:
+        ws = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        idx = torch.empty(k, dtype=torch.int64, device="cuda")
+        gs.gs_sketch_insert(sk, 0, _dev(_prune_input(rng, d, k, False)), d)
+        gs.gs_sketch_merge_tree(sk, 1)
+        gs.gs_query_topk(sk, d, k, idx, None, ws)
+        torch.cuda.synchronize()
+        e_int = H.host(ws[: 4 * d].view(torch.float32)).copy()
+        pruned, n = H.pruned_rows(e_int, r)
+        # markers name f <= n < r rows, so for r = 4 every one names 3
+        assert pruned.mean() > 0.5 and (r - 1 == f or np.any(n > f)), "coordinates should stop at several row counts"
+        T = np.empty(r * c, np.float32)
+        gs.gs_sketch_copy_to_host(sk, -1, T)
+        T = T.reshape(r, c)
+        bk = torch.empty(r * d, dtype=torch.int32, device="cuda")
+        sg = torch.empty(r * d, dtype=torch.int8, device="cuda")
+        gs.gs_hash_eval(sk, _dev(np.arange(d, dtype=np.int64)), d, bk, sg)
+        bk, sg = H.host(bk).reshape(r, d), H.host(sg).reshape(r, d)
+        v = T[np.arange(r)[:, None], bk] * sg.astype(np.float32)   # exact: a sign flip
+        lo, hi = 0.0, np.inf            # the prune key must satisfy lo < t <= hi
+        for rows in range(f, r + 1):
+            at = np.nonzero(pruned)[0][n == rows] if rows < r else np.nonzero(~pruned)[0]
+            if at.size == 0:
+                continue
+            if rows < r:
+                lo = max(lo, float(_settle_threshold(v[:rows, at], f).max()))
+            if rows > f:
+                hi = min(hi, float(_settle_threshold(v[:rows - 1, at], f).min()))
+        assert lo < hi, f"no prune key explains the rows read: settled below {lo}, unsettled from {hi}"
+    finally:
+        gs.gs_sketch_destroy(sk)
 
 
 def test_no_pruning_below_4m_coordinates(gs, H):
@@ -719,7 +772,7 @@ def test_heavymix_pruned_matches_full(gs, H, r, k, spikes):
         l2h = H.host(l2)
         assert abs(l2h[0] - l2h[1]) <= 1e-12 * l2h[0]   # fp64 atomic sums: order varies
         assert np.array_equal(H.host(idx_full), oracle.heavymix_select(H.host(est), float(l2h[0]), k, fill_seed))
-        pruned = e_int.view(np.uint32) == np.uint32(0x80000000)
+        pruned, _ = H.pruned_rows(e_int, r)
         assert pruned.mean() > 0.2, "rows were not skipped"
         e = H.host(est).astype(np.float64)
         assert np.all(e[pruned] ** 2 < l2h[0] / k)
