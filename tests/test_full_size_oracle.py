@@ -39,7 +39,7 @@ def test_parallel_oracle_equals_plain_step(monkeypatch):
         assert np.allclose(band, oracle.cell_band(res.merged_abs, co, np.arange(d)), rtol=1e-13, atol=0)
         assert np.array_equal(oracle.topk_by_threshold(est, k), res.idx)
         # one slot alone, its pieces split over both processes: the same result
-        T0, A0, own0, e0, c0 = po.workers([0], rho, res.idx, tabled=[0])
+        T0, _, own0, e0, c0 = po.workers([0], rho, res.idx, tabled=[0])
         assert np.allclose(own0[0][0], own[0][0], rtol=0, atol=1e-12 * res.abs_tables[0].max())
         assert np.allclose(T0, own[0][0], rtol=0, atol=1e-12 * res.abs_tables[0].max())
         assert np.array_equal(e0[0], e_sel[0]) and c0[0] == [0, 0, 0]

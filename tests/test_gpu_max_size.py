@@ -59,7 +59,7 @@ def test_step_at_max_dimension(gs):
         table = np.empty(r * c, dtype=np.float32)
         gs.gs_sketch_copy_to_host(sk, -1, table)
         coeffs = oracle.derive_coefficients(r, seed)
-        T, A = oracle.sketch_sparse(spikes, vals.astype(np.float64), coeffs, c)
+        T, _ = oracle.sketch_sparse(spikes, vals.astype(np.float64), coeffs, c)
         assert np.array_equal(table.reshape(r, c).astype(np.float64), T)  # a few exact fp32 sums
 
         rest = np.setdiff1d(np.arange(k, dtype=np.int64), spikes)[: k - spikes.size]

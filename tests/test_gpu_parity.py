@@ -807,7 +807,7 @@ def test_heavymix(gs, H, d, r, c, k, spikes, scale):
         assert np.array_equal(idx, oracle.heavymix_select(est, l2sq, k, fill_seed))
         # against the fp64 oracle: the same l2sq within the cell tolerance, est within its band
         T, A = oracle.sketch(x, coeffs, c)
-        idx_o, est_o, l2_o = oracle.heavymix(T, coeffs, d, k, fill_seed)
+        _, est_o, l2_o = oracle.heavymix(T, coeffs, d, k, fill_seed)
         assert abs(l2sq - l2_o) <= 1e-4 * l2_o
         band = oracle.cell_band(A, coeffs, np.arange(d))
         assert np.all(np.abs(est.astype(np.float64) - est_o) <= band)

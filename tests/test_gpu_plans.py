@@ -372,7 +372,7 @@ def test_heavymix_step_and_plan(gs, H):
             tabs = [oracle.sketch(e1, coeffs, c, hashes) for _, e1 in pre]
             T = oracle.merge_tree([a for a, _ in tabs])
             A = oracle.merge_tree([b for _, b in tabs])
-            idx_o, est_o, l2_o = oracle.heavymix(T, coeffs, d, k, fill_seed, hashes)
+            _, est_o, l2_o = oracle.heavymix(T, coeffs, d, k, fill_seed, hashes)
             band = oracle.cell_band(A, coeffs, np.arange(d))
             assert np.all(np.abs(est.astype(np.float64) - est_o) <= band)
             assert abs(l2sq - l2_o) <= 1e-4 * l2_o

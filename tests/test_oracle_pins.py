@@ -132,7 +132,7 @@ def test_sketch_linearity_exact(r, c):
     rng = np.random.default_rng(r * c)
     co = oracle.derive_coefficients(r, 99 + c)
     x1, x2 = _dyadic(rng, 5000), _dyadic(rng, 5000)
-    T1, A1 = oracle.sketch(x1, co, c)
+    T1, _ = oracle.sketch(x1, co, c)
     T2, _ = oracle.sketch(x2, co, c)
     T12, _ = oracle.sketch(x1 + x2, co, c)   # x1 + x2 exact in fp32 for these values
     assert np.array_equal(T1 + T2, T12)
@@ -433,7 +433,7 @@ def test_heavymix_h_bound_and_large_h_branch():
 def test_heavymix_random_fill_brute_force():
     co, x, T = _heavymix_fixture(2)
     d, k, seed = x.size, 200, 12345
-    idx, est, l2sq = oracle.heavymix(T, co, d, k, fill_seed=seed)
+    idx, _, l2sq = oracle.heavymix(T, co, d, k, fill_seed=seed)
     h = [i for i in range(d) if float(x[i]) ** 2 >= l2sq / k]
     assert len(h) < k
     xi = {i: int(oracle.splitmix64_at(seed, [i])[0]) >> 33 for i in range(d)}

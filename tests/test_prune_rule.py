@@ -65,7 +65,7 @@ def test_even_r_mean_stays_below_the_threshold():
 def test_unsettled_rows_can_reach_the_threshold():
     """The rule is not loose in the other direction: with f - 1 cells below t after the first
     f rows, the unread cells decide, and the median can reach t."""
-    r, f = 5, 3
+    f = 3   # r = 5
     t = np.float32(1.0)
     read = np.array([0.1, -0.2, 2.0], np.float32)
     assert not settled(read, t, f)
