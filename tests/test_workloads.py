@@ -46,3 +46,23 @@ def test_spikes_shared_across_workers():
     g0 = W.make_gradient(w, 0, 0)
     g1 = W.make_gradient(w, 1, 3)
     assert np.all(np.sign(g0[pos]) == sgn) and np.all(np.sign(g1[pos]) == sgn)
+
+
+def test_device_draw_follows_the_block_recipe():
+    """The device-side draw (here on the CPU generator): seeded per (step, worker), and each
+    block's entries have the block's scale."""
+    import torch
+    w = W.get_config("resnet18")
+    a = W.make_gradient_torch(w, 1, 2, torch.empty(w.d))
+    b = W.make_gradient_torch(w, 1, 2, torch.empty(w.d))
+    c = W.make_gradient_torch(w, 1, 3, torch.empty(w.d))
+    assert torch.equal(a, b) and not torch.equal(a, c)
+    x = a.numpy().astype(np.float64)
+    off = 0
+    for n, s in zip(w.blocks, W.block_scales(w)):
+        if n >= 20_000:
+            sd = x[off:off + n].std()
+            assert abs(sd / s - 1) < 0.05, (n, s, sd)
+            assert abs(x[off:off + n].mean()) < 5 * s / np.sqrt(n)
+        off += n
+    assert off == w.d
