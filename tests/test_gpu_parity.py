@@ -449,7 +449,7 @@ def _settle_threshold(v, f):
     return np.maximum(srt[f - 1], -srt[v.shape[0] - f])
 
 
-@pytest.mark.parametrize("r", [4, 5, 7])
+@pytest.mark.parametrize("r", [3, 4, 5, 7, 16])
 def test_pruned_rows_follow_the_rule(gs, H, r):
     """The rows each coordinate read, from its marker, against the rule, with the signed cells
     recomputed on the host from the merged table and the hash values: one prune key t must
