@@ -521,6 +521,9 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
     }
     q = None
     q_ms = ph["query"]
+    with_selection = q_ms is None and ph["query_select"] is not None   # eager: one pair of events per call
+    if with_selection:
+        q_ms = ph["query_select"]
     if q_ms is not None and variant != "heavymix":
         prunes = d >= PRUNE_MIN_DIM and r >= 3 and (w.c & (w.c - 1)) == 0
         nq = (d + 3) // 4
@@ -529,7 +532,8 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
         g_ms = probes.get("query_ms")
         ach = requests / (q_ms / 1e3) / 1e9
         q = {
-            "kernel": f"k_qsample + k_query<{r}> + k_repair (median query, S4)" if prunes else f"k_query<{r}> (S4)",
+            "kernel": (f"k_qsample + k_query<{r}> + k_repair (median query, S4)" if prunes else f"k_query<{r}> (S4)") +
+                      (" and the S5 selection: eager, timed around the gs_query_topk call" if with_selection else ""),
             "bound": "L1->L2 requests (scattered 4-byte reads of the merged table)",
             "avg_ms": round(q_ms, 4), "pruned_fraction": round(pruned, 4), "rows_read_per_coord": round(rows_read, 3),
             "requests_per_step": requests, "requests_per_coord": round(requests / d, 3),
@@ -541,6 +545,8 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
             "hbm": {"algorithmic_bytes": 4 * d, "achieved_GBps": round(4 * d / (q_ms / 1e3) / 1e9, 1),
                     "frac": round(4 * d / (q_ms / 1e3) / 1e9 / peaks["hbm_gbs"], 4)},
             "select_ms": None if ph["select"] is None else round(ph["select"], 4),
+            "timed": "query and selection together (eager call)" if with_selection else
+                     "query only (event nodes inside the step's graph)",
         }
     return k1, q
 
@@ -660,7 +666,7 @@ def short_summary(res: dict, w) -> dict:
                                           "rows_read_per_coord": q["rows_read_per_coord"],
                                           "achieved_G_requests_per_s": q["achieved_G_requests_per_s"],
                                           "peak_G_requests_per_s": q["peak_G_requests_per_s"], "frac": q["frac"],
-                                          "select_ms": q["select_ms"]},
+                                          "select_ms": q["select_ms"], "timed": q["timed"]},
         "gpu_launches_per_step": res["gpu_launches_per_step"],
     }
     for key in ("streaming", "ms_per_step_without_generation", "query_and_selection_ms"):
