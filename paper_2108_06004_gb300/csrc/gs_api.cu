@@ -419,8 +419,7 @@ gs_status check_host_step(gs_sketch* sk, float* const* momentum, float* const* e
 // Where the fused kernel reads each worker's host gradient: the gradient itself where the GPU
 // can address it (pinned or registered host memory, device memory, or any host memory when
 // the device has pageable-memory access), else nullptr: first copied into grad_dev[p].
-void host_sources(const gs_sketch* sk, const float* const* grad_host, float* const* grad_dev,
-                  std::vector<const float*>& src) {
+void host_sources(const gs_sketch* sk, const float* const* grad_host, std::vector<const float*>& src) {
   int pageable = 0;
   cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, sk->device);
   src.assign((size_t)sk->workers, nullptr);
@@ -1103,7 +1102,7 @@ gs_status gs_step_host(gs_sketch* sk, float* const* momentum, float* const* erro
   GS_TRY(check_host_step(sk, momentum, error, grad_host, grad_dev, d, k, idx_host, vals_host, workspace,
                          workspace_bytes));
   std::vector<const float*> src;
-  host_sources(sk, grad_host, grad_dev, src);
+  host_sources(sk, grad_host, src);
   cudaStream_t s = as_stream(stream);
   GS_TRY(host_step_enqueue(sk, momentum, error, grad_host, grad_dev, src, d, rho, k, idx_host, vals_host, workspace, s));
   cudaError_t e = cudaStreamSynchronize(s);
@@ -1159,7 +1158,7 @@ gs_status gs_step_host_plan_create(gs_sketch* sk, float* const* momentum, float*
   GS_TRY(check_host_step(sk, momentum, error, grad_host, grad_dev, d, k, idx_host, vals_host, workspace,
                          workspace_bytes));
   std::vector<const float*> src;
-  host_sources(sk, grad_host, grad_dev, src);
+  host_sources(sk, grad_host, src);
   return capture_plan(sk->device, flags, plan_out, [&](cudaStream_t s, InsertMarks marks) {
     return host_step_enqueue(sk, momentum, error, grad_host, grad_dev, src, d, rho, k, idx_host, vals_host, workspace,
                              s, marks);
