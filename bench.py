@@ -45,6 +45,13 @@ L2_BYTES = 126 << 20     # GB300 L2; inputs below twice this are flushed between
 PER_CONFIG_STEPS = {"tiny-2^20": 300, "resnet18": 300, "resnet50": 100, "vgg16": 5, "bert-large": 3}
 PRUNE_MIN_DIM = 1 << 22  # the library skips query rows from this dimension on
 SAMPLE_PERIOD = 256      # ... with a prune-key sample of the first four of every 256 coordinates
+CLASS_BYTES = 192 << 10  # ... and classifies the first r/2 + 1 rows in shared memory when they fit
+
+
+def query_classifies(r: int, c: int) -> bool:
+    """Whether a pruning query of r rows and c columns runs the shared-memory classification
+    (one more kernel, which writes the cell classes)."""
+    return 3 <= r <= 16 and c >= 64 and (c & (c - 1)) == 0 and (r // 2 + 1) * c // 4 <= CLASS_BYTES
 
 VARIANTS = {
     "error_feedback": "S1-S6: per-worker momentum and error vectors, exact second round",
@@ -394,15 +401,19 @@ class Runner:
                 "gen": mean(per_step("gen")), "n": len(ins)}
 
     def query_rows(self):
-        """(fraction of coordinates that stopped early, rows read per coordinate) in the last
-        query: a coordinate that stopped after n rows leaves -(n * 2^-149) as its estimate."""
+        """(fraction of coordinates that stopped early, rows examined per coordinate, table
+        cells read per coordinate) in the last query: a coordinate that stopped after examining
+        n rows, g of whose cells it read from the table, leaves -((32 g + n) * 2^-149) as its
+        estimate; every other coordinate read all r cells."""
         import torch
         d, r = self.w.d, self.w.r
         bits = self.ws[: 4 * d].view(torch.int32)
-        marked = (bits > -2**31) & (bits <= -2**31 + 16)
+        marked = (bits > -2**31) & (bits < -2**31 + 1024)
         n_marked = int(marked.sum().item())
-        rows_marked = int((bits[marked].to(torch.int64) + 2**31).sum().item())
-        return n_marked / d, (rows_marked + (d - n_marked) * r) / d
+        low = bits[marked].to(torch.int64) + 2**31
+        examined = int((low & 31).sum().item())
+        gathered = int((low >> 5).sum().item())
+        return n_marked / d, (examined + (d - n_marked) * r) / d, (gathered + (d - n_marked) * r) / d
 
     def close(self):
         for plan in self.plans:
@@ -423,7 +434,8 @@ def launches_per_step(run: Runner, variant: str) -> int:
     if variant == "heavymix":
         query = 3 + 6                                 # sumsq, theta, query (with the keys) + selection
     else:
-        query = 1 + 6 + (2 if prunes else 0)          # query + selection (+ sample and repair check)
+        # query + selection (+ sample and repair check, + the cell classes)
+        query = 1 + 6 + (2 + int(query_classifies(w.r, w.c)) if prunes else 0)
     tail = 6 if variant == "sketched_state" else 1
     return inserts + 1 + query + tail
 
@@ -474,7 +486,7 @@ def time_steps(run: Runner, steps: int, warmup: int, world: int, dev, sampler=No
 
 
 def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dict, pruned: float,
-              rows_read: float):
+              rows_read: float, cells_read: float):
     """The insert-phase roofline (HBM, with the measured request ceiling as co-bound) and the
     median query's (L1->L2 requests against the measured gather ceiling; HBM bytes alongside)."""
     w = run.w
@@ -528,14 +540,17 @@ def rooflines(run: Runner, variant: str, ph: dict, peaks, peak_kind, probes: dic
         prunes = d >= PRUNE_MIN_DIM and r >= 3 and (w.c & (w.c - 1)) == 0
         nq = (d + 3) // 4
         n_s = 4 * ((nq + SAMPLE_PERIOD // 4 - 1) // (SAMPLE_PERIOD // 4)) if prunes else 0
-        requests = d * rows_read + n_s * r
+        requests = d * cells_read + n_s * r
         g_ms = probes.get("query_ms")
         ach = requests / (q_ms / 1e3) / 1e9
         q = {
-            "kernel": (f"k_qsample + k_query<{r}> + k_repair (median query, S4)" if prunes else f"k_query<{r}> (S4)") +
+            "kernel": ((f"k_qsample + k_pbits + k_query_bits<{r}> + k_repair (median query, S4)"
+                        if query_classifies(r, w.c) else f"k_qsample + k_query<{r}> + k_repair (median query, S4)")
+                       if prunes else f"k_query<{r}> (S4)") +
                       (" and the S5 selection: eager, timed around the gs_query_topk call" if with_selection else ""),
             "bound": "L1->L2 requests (scattered 4-byte reads of the merged table)",
-            "avg_ms": round(q_ms, 4), "pruned_fraction": round(pruned, 4), "rows_read_per_coord": round(rows_read, 3),
+            "avg_ms": round(q_ms, 4), "pruned_fraction": round(pruned, 4), "rows_examined_per_coord": round(rows_read, 3),
+            "cells_read_per_coord": round(cells_read, 3),
             "requests_per_step": requests, "requests_per_coord": round(requests / d, 3),
             "achieved_G_requests_per_s": round(ach, 1),
             "peak_G_requests_per_s": None if g_ms is None else round(d * r / (g_ms / 1e3) / 1e9, 1),
@@ -582,9 +597,10 @@ def measure(gs, w, variant, eager, steps, warmup, world, rank, dev, stream, peak
     torch.cuda.synchronize()
     elapsed_ms, n_warm, n_by_plan = time_steps(run, steps, warmup, world, dev, sampler, flush)
     ph = run.phase_times(n_by_plan)
-    pruned, rows_read = run.query_rows() if variant != "heavymix" else (0.0, float(run.w.r))
+    pruned, rows_read, cells_read = run.query_rows() if variant != "heavymix" else (0.0, float(run.w.r),
+                                                                                     float(run.w.r))
     pr = probe_ceilings(run) if probes else {}
-    k1, q = rooflines(run, variant, ph, peaks, peak_kind, pr, pruned, rows_read)
+    k1, q = rooflines(run, variant, ph, peaks, peak_kind, pr, pruned, rows_read, cells_read)
     value = whole_job_rate(world, w.P, w.d, steps, elapsed_ms / 1e3)
     res = {
         "value": value, "ms_per_step": round(elapsed_ms / steps, 4), "steps": steps, "warmup_steps_run": n_warm,
@@ -663,7 +679,8 @@ def short_summary(res: dict, w) -> dict:
                    "request_ceiling_ms": k1["co_bound"]["peak_ms"], "frac_of_request_ceiling": k1["co_bound"]["frac"],
                    "request_ceiling_frac_of_hbm": k1["co_bound"]["peak_frac_of_hbm"]},
         "query": None if q is None else {"avg_ms": q["avg_ms"], "pruned_fraction": q["pruned_fraction"],
-                                          "rows_read_per_coord": q["rows_read_per_coord"],
+                                          "rows_examined_per_coord": q["rows_examined_per_coord"],
+                                          "cells_read_per_coord": q["cells_read_per_coord"],
                                           "achieved_G_requests_per_s": q["achieved_G_requests_per_s"],
                                           "peak_G_requests_per_s": q["peak_G_requests_per_s"], "frac": q["frac"],
                                           "select_ms": q["select_ms"], "timed": q["timed"]},

@@ -66,6 +66,24 @@ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 __device__ __forceinline__ uint32_t key_of(float v) { return __float_as_uint(v) & 0x7FFFFFFFu; }
 
+// The query's hash arithmetic, without compares (the query is bound by its integer work).
+// For s < 2^62 - 1, s mod p is s - p when s >= p and s otherwise; s >= p exactly when bit 61
+// of s + 1 is set, and then s - p = (s + 1) - 2^61 = (s + 1) & p.  So for s < 2p:
+//   s mod p = (s + ((s + 1) >> 61)) & p.
+__device__ __forceinline__ uint64_t reduce61(uint64_t s) { return (s + ((s + 1) >> 61)) & kP61; }
+
+// x + a mod p for x, a < p (the incremental form of the hash): the same value as step61.
+__device__ __forceinline__ uint64_t step61_nb(uint64_t x, uint64_t a) { return reduce61(x + a); }
+
+// (a*i + b) mod p for a, b < p and i < 2^32: the same value as affine61.  The sum of the
+// partial products is below 3 * 2^61; one fold leaves it at most p + 2, then reduce61.
+__device__ __forceinline__ uint64_t affine61_nb(uint64_t a, uint64_t b, uint32_t i) {
+  const uint64_t p0 = (uint64_t)(uint32_t)a * i;
+  const uint64_t p1 = (uint64_t)(uint32_t)(a >> 32) * i;
+  const uint64_t s = (p1 >> 29) + ((p1 & ((1ull << 29) - 1)) << 32) + fold61(p0) + b;
+  return reduce61(fold61(s));
+}
+
 // Warp-aggregated shared-memory histogram update; every lane of the warp must call it.
 __device__ __forceinline__ void hist_add(uint32_t* sh, uint32_t bin) {
   const uint32_t peers = __match_any_sync(kFull, bin);
@@ -238,11 +256,17 @@ struct QueryParams {
 // the query's own selection state, so every CTA of k_query and k_repair reads the same value.
 // It is a level-1 bin edge: whether it was safe is then exactly whether the level-1 pick
 // lands in its bin or above, which k_repair checks.
-// A coordinate that stopped early stores -(n * 2^-149), n = the rows it read (f <= n < r):
-// a key in level-1 bin 0 that k_repair recognises and the measurement can count.
-constexpr uint32_t kPrunedBits = 0x80000000u;  // sign bit; the low bits hold the rows read
+// A coordinate that stopped early stores the marker -((32 g + n) * 2^-149): n = the rows whose
+// cells it examined (f <= n < r), g = how many of those cells it read from the table (g = n
+// when every examined cell is read).  It is a key in level-1 bin 0 that k_repair recognises
+// and the measurement can count.
+constexpr uint32_t kPrunedBits = 0x80000000u;  // sign bit; the low bits hold n and g
 
-__device__ __forceinline__ bool is_pruned(uint32_t bits) { return bits - (kPrunedBits + 1u) < (uint32_t)GS_MAX_ROWS; }
+__device__ __forceinline__ uint32_t pruned_marker(int examined, int gathered) {
+  return kPrunedBits | ((uint32_t)gathered << 5) | (uint32_t)examined;
+}
+
+__device__ __forceinline__ bool is_pruned(uint32_t bits) { return bits - (kPrunedBits + 1u) < 0x3FFu; }
 
 // Counts of a coordinate's cells below t (lt) and above -t (gt), on keys: |v| < t is
 // key_of(v) < pk; a NaN counts on neither side.
@@ -295,16 +319,16 @@ __global__ void __launch_bounds__(kBlock, R <= 7 ? 4 : 1) k_query(const __grid_c
       float v[4][R];
 #pragma unroll
       for (int j = 0; j < kF; ++j) {
-        uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
-        uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
+        uint64_t x = affine61_nb(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+        uint64_t y = affine61_nb(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
         const float* row = prm.T + (size_t)j * prm.c;
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           v[t][j] = 0.f;
           if (t < tmax) {
             v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
-            x = step61(x, prm.h.a[j]);
-            y = step61(y, prm.h.a2[j]);
+            x = step61_nb(x, prm.h.a[j]);
+            y = step61_nb(y, prm.h.a2[j]);
           }
         }
       }
@@ -322,8 +346,8 @@ __global__ void __launch_bounds__(kBlock, R <= 7 ? 4 : 1) k_query(const __grid_c
       }
 #pragma unroll
       for (int j = kF; j < R; ++j) {
-        uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
-        uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
+        uint64_t x = affine61_nb(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+        uint64_t y = affine61_nb(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
         const float* row = prm.T + (size_t)j * prm.c;
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
@@ -334,8 +358,8 @@ __global__ void __launch_bounds__(kBlock, R <= 7 ? 4 : 1) k_query(const __grid_c
               tally(v[t][j], pk, lt[t], gt[t]);
               ++rows[t];
             }
-            x = step61(x, prm.h.a[j]);
-            y = step61(y, prm.h.a2[j]);
+            x = step61_nb(x, prm.h.a[j]);
+            y = step61_nb(y, prm.h.a2[j]);
           }
         }
         if (j + 1 < R) {
@@ -345,7 +369,7 @@ __global__ void __launch_bounds__(kBlock, R <= 7 ? 4 : 1) k_query(const __grid_c
       }
 #pragma unroll
       for (int t = 0; t < 4; ++t)
-        m[t] = done[t] ? __uint_as_float(kPrunedBits | (uint32_t)rows[t]) : median_of<R>(v[t]);
+        m[t] = done[t] ? __uint_as_float(pruned_marker(rows[t], rows[t])) : median_of<R>(v[t]);
       store_est(prm, i0, tmax, m);
       if (HM) {
 #pragma unroll
@@ -368,6 +392,152 @@ __global__ void __launch_bounds__(kBlock, R <= 7 ? 4 : 1) k_query(const __grid_c
     hist_flush(sh, prm.hist, kBins);
     last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
   }
+}
+
+// ---- the pruning query with the first rows classified in shared memory ---------------------
+// The settle rule needs, for each of the first f = r/2 + 1 cells of a coordinate, only which side
+// of the prune key t its value lies on.  For a row that is a class per table cell: 0 (|T| < t),
+// 1 (T >= t), 2 (T <= -t) or 3 (NaN); the sign hash of the coordinate swaps classes 1 and 2.
+// Where the classes of the first f rows fit in shared memory (2 bits per cell), k_pbits writes
+// them once per query and k_query_bits looks them up instead of reading those cells from L2.  A
+// coordinate that settles within the first f rows then reads no cell at all; one that examines
+// later rows reads those cells as k_query does; one that does not settle reads every cell for
+// its full median.  The rows examined, the stops and the estimates are the same as k_query's.
+constexpr uint32_t kBitsBytes = 192u << 10;   // dynamic shared memory for the classes
+
+constexpr int kBitsBlock = 1024;              // one CTA of 32 warps per SM
+
+__device__ __forceinline__ uint32_t cell_class(float v, uint32_t pk) {
+  const uint32_t b = __float_as_uint(v), key = b & 0x7FFFFFFFu;
+  if (key > 0x7F800000u) return 3u;
+  if (key < pk) return 0u;
+  return (b >> 31) ? 2u : 1u;
+}
+
+// Word w holds the classes of cells 16 w .. 16 w + 15 of the first rows of the row-major merged
+// table, cell 16 w + u at bits 2u, 2u + 1.  nwords = f * c / 16.
+__global__ void __launch_bounds__(kBlock) k_pbits(const float* __restrict__ T, int64_t nwords,
+                                                  const SelectState* st, uint32_t* __restrict__ words) {
+  grid_begin();
+  const uint32_t pk = __ldcg(&st->prune_key);
+  for (int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; w < nwords; w += (int64_t)gridDim.x * blockDim.x) {
+    const float4* src = reinterpret_cast<const float4*>(T) + 4 * w;
+    uint32_t out = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 v = __ldg(src + q);
+      out |= (cell_class(v.x, pk) | cell_class(v.y, pk) << 2 | cell_class(v.z, pk) << 4 | cell_class(v.w, pk) << 6)
+             << (8 * q);
+    }
+    words[w] = out;
+  }
+}
+
+template <int R>
+__global__ void __launch_bounds__(kBitsBlock, 1) k_query_bits(const __grid_constant__ QueryParams prm,
+                                                              const uint32_t* __restrict__ words) {
+  grid_begin();
+  extern __shared__ uint4 sbits4[];
+  const uint32_t* sbits = reinterpret_cast<const uint32_t*>(sbits4);
+  __shared__ uint32_t sh[kBins];
+  constexpr int kF = R / 2 + 1;
+  {
+    const int64_t n4 = (int64_t)kF * (prm.c / 16) / 4;
+    const uint4* src = reinterpret_cast<const uint4*>(words);
+    for (int64_t w = threadIdx.x; w < n4; w += blockDim.x) sbits4[w] = __ldcg(src + w);
+  }
+  for (int b = threadIdx.x; b < kBins; b += blockDim.x) sh[b] = 0;
+  __syncthreads();
+  const int64_t d = prm.d, nq = (d + 3) / 4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int lane = threadIdx.x & 31;
+  const uint32_t pk = prune_key_of(prm);
+  for (int64_t q0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); q0 < nq; q0 += stride) {
+    const int64_t q = q0 + lane;
+    const int64_t i0 = q * 4;
+    const int tmax = q < nq ? (d - i0 < 4 ? (int)(d - i0) : 4) : 0;
+    float m[4] = {0.f, 0.f, 0.f, 0.f};
+    if (tmax > 0) {
+      float v[4][R];
+      uint32_t cell[4][kF];  // bucket of each of the first kF rows, sign bit of the cell in bit 31
+      int lt[4], gt[4], rows[4];
+      bool done[4];
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        lt[t] = 0;
+        gt[t] = 0;
+      }
+      // the first kF rows: classes from shared memory, no table reads
+#pragma unroll
+      for (int j = 0; j < kF; ++j) {
+        uint64_t x = affine61_nb(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+        uint64_t y = affine61_nb(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          cell[t][j] = 0u;
+          if (t < tmax) {
+            const uint32_t b = (uint32_t)x & prm.cmask;
+            const uint32_t g = (uint32_t)j * prm.c + b;
+            uint32_t cls = (sbits[g >> 4] >> ((g & 15u) * 2u)) & 3u;
+            if ((uint32_t)y & 1u) cls = (cls == 1u || cls == 2u) ? (3u - cls) : cls;
+            lt[t] += (cls == 0u || cls == 2u) ? 1 : 0;
+            gt[t] += (cls == 0u || cls == 1u) ? 1 : 0;
+            cell[t][j] = b | signbit_of(y);
+            x = step61_nb(x, prm.h.a[j]);
+            y = step61_nb(y, prm.h.a2[j]);
+          }
+        }
+      }
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        rows[t] = kF;
+        done[t] = pk != 0u && lt[t] >= kF && gt[t] >= kF;
+      }
+      // the later rows, each only while the coordinate is undecided (read from the table)
+#pragma unroll
+      for (int j = kF; j < R; ++j) {
+        uint64_t x = affine61_nb(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+        uint64_t y = affine61_nb(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
+        const float* row = prm.T + (size_t)j * prm.c;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          v[t][j] = 0.f;
+          if (t < tmax) {
+            if (!done[t]) {
+              v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
+              tally(v[t][j], pk, lt[t], gt[t]);
+              ++rows[t];
+            }
+            x = step61_nb(x, prm.h.a[j]);
+            y = step61_nb(y, prm.h.a2[j]);
+          }
+        }
+        if (j + 1 < R) {
+#pragma unroll
+          for (int t = 0; t < 4; ++t) done[t] = done[t] || (pk != 0u && lt[t] >= kF && gt[t] >= kF);
+        }
+      }
+      // a coordinate that did not settle needs its full median: read its first kF cells now
+#pragma unroll
+      for (int j = 0; j < kF; ++j) {
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          v[t][j] = 0.f;
+          if (t < tmax && !done[t])
+            v[t][j] = apply_sign(__ldg(prm.T + (size_t)j * prm.c + (cell[t][j] & 0x7FFFFFFFu)),
+                                 cell[t][j] & 0x80000000u);
+        }
+      }
+#pragma unroll
+      for (int t = 0; t < 4; ++t)
+        m[t] = done[t] ? __uint_as_float(pruned_marker(rows[t], rows[t] - kF)) : median_of<R>(v[t]);
+      store_est(prm, i0, tmax, m);
+    }
+#pragma unroll
+    for (int t = 0; t < 4; ++t) hist_add(sh, t < tmax ? (key_of(m[t]) >> kL1Shift) : kNone);
+  }
+  hist_flush(sh, prm.hist, kBins);
+  last_block_pick(prm.hist, 11, prm.st, 0, prm.k);
 }
 
 // Runs after k_query.  If the level-1 pick landed in the prune key's bin or above, the k-th
@@ -440,16 +610,16 @@ __global__ void __launch_bounds__(kBlock) k_qsample(const __grid_constant__ Quer
       float v[4][R];
 #pragma unroll
       for (int j = 0; j < R; ++j) {
-        uint64_t x = affine61(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
-        uint64_t y = affine61(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
+        uint64_t x = affine61_nb(prm.h.a[j], prm.h.b[j], (uint32_t)i0);
+        uint64_t y = affine61_nb(prm.h.a2[j], prm.h.b2[j], (uint32_t)i0);
         const float* row = prm.T + (size_t)j * prm.c;
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           v[t][j] = 0.f;
           if (t < tmax) {
             v[t][j] = apply_sign(__ldg(row + ((uint32_t)x & prm.cmask)), signbit_of(y));
-            x = step61(x, prm.h.a[j]);
-            y = step61(y, prm.h.a2[j]);
+            x = step61_nb(x, prm.h.a[j]);
+            y = step61_nb(y, prm.h.a2[j]);
           }
         }
       }
@@ -1057,6 +1227,50 @@ struct QueryTable {
 template <int... Rs>
 constexpr QueryLauncher QueryTable<Rs...>::table[sizeof...(Rs)];
 
+// k_query_bits<R> for a pruning query whose first rows' classes fit kBitsBytes: the classes are
+// written into `words` (f * c / 4 bytes of scratch) first.
+template <int R>
+cudaError_t launch_query_bits_r(const QueryParams& p, uint32_t* words, cudaStream_t s) {
+  constexpr int kF = R / 2 + 1;
+  const int64_t nwords = (int64_t)kF * (p.c / 16);
+  const int gw = (int)((nwords + kBlock - 1) / kBlock);
+  launch(k_pbits, gw, kBlock, s, p.T, nwords, p.st, words);
+  auto kern = k_query_bits<R>;
+  const size_t smem = (size_t)nwords * sizeof(uint32_t);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const int64_t need = ((p.d + 3) / 4 + kBitsBlock - 1) / kBitsBlock;
+  const int grid = (int)(need < device_info().sms ? (need < 1 ? 1 : need) : device_info().sms);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kBitsBlock);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, p, (const uint32_t*)words);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+typedef cudaError_t (*BitsLauncher)(const QueryParams&, uint32_t*, cudaStream_t);
+
+template <int... Rs>
+struct BitsTable {
+  static constexpr BitsLauncher table[sizeof...(Rs)] = {&launch_query_bits_r<Rs>...};
+};
+template <int... Rs>
+constexpr BitsLauncher BitsTable<Rs...>::table[sizeof...(Rs)];
+
+// Whether a pruning query of r rows and c (a power of two) columns classifies its first rows in
+// shared memory.
+bool query_uses_bits(int r, uint32_t c) {
+  const uint64_t bytes = (uint64_t)(r / 2 + 1) * c / 4;
+  return r >= 3 && r <= GS_MAX_ROWS && is_pow2(c) && c >= 64 && bytes <= kBitsBytes;
+}
+
 template <int R>
 cudaError_t launch_repair_r(const QueryParams& p, uint32_t* hist_r, cudaStream_t s) {
   auto kern = k_repair<R>;
@@ -1257,7 +1471,13 @@ cudaError_t launch_query_topk(const float* merged, const HashCoeffs& h, int r, u
     using T = SampleTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
     if ((err = T::table[r - 1](qp, w.hist + 4 * kBins, j_target, s)) != cudaSuccess) return err;
   }
-  if ((err = launch_query(qp, s)) != cudaSuccess) return err;
+  if (qp.prune && query_uses_bits(r, c)) {
+    // the classes go in the candidate area, which the selection only uses after the query
+    using T = BitsTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
+    if ((err = T::table[r - 1](qp, reinterpret_cast<uint32_t*>(w.cand), s)) != cudaSuccess) return err;
+  } else if ((err = launch_query(qp, s)) != cudaSuccess) {
+    return err;
+  }
   if (qp.prune) {
     using T = RepairTable<1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15, 16>;
     if ((err = T::table[r - 1](qp, w.hist + 3 * kBins, s)) != cudaSuccess) return err;

@@ -68,12 +68,17 @@ def host(t: torch.Tensor) -> np.ndarray:
 
 
 def pruned_rows(e_int: np.ndarray, r: int):
-    """(mask, rows): the coordinates whose workspace estimate is a pruning marker, -(n * 2^-149)
-    with n the rows read, and n for each of them.  Every marker must name r/2 + 1 <= n < r."""
+    """(mask, rows): the coordinates whose workspace estimate is a pruning marker,
+    -((32 g + n) * 2^-149) with n the rows whose cells were examined and g how many of those
+    cells were read from the table, and n for each of them.  Every marker must name
+    f <= n < r (f = r/2 + 1) and n - f <= g <= n."""
     bits = e_int.view(np.uint32)
-    mask = (bits > np.uint32(0x80000000)) & (bits <= np.uint32(0x80000010))
-    n = (bits[mask] & np.uint32(0xFF)).astype(np.int64)
-    assert np.all((n >= r // 2 + 1) & (n < r)), "a marker names an impossible row count"
+    mask = (bits > np.uint32(0x80000000)) & (bits < np.uint32(0x80000400))
+    n = (bits[mask] & np.uint32(31)).astype(np.int64)
+    g = ((bits[mask] >> np.uint32(5)) & np.uint32(31)).astype(np.int64)
+    f = r // 2 + 1
+    assert np.all((n >= f) & (n < r)), "a marker names an impossible row count"
+    assert np.all((g <= n) & (g >= n - f)), "a marker names an impossible count of cells read"
     return mask, n
 
 
