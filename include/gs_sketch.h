@@ -172,8 +172,11 @@ gs_status gs_query_topk_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, the query may skip rows.  Rows
  * are read in order, and a coordinate stops once, with f = r/2 + 1, at least f of the cells
  * read are below a threshold t and at least f are above -t: then |est| < t whatever the
- * other rows hold, and it cannot be selected.  Its estimate is left in the workspace as
- * -(n * 2^-149), n the rows it read (f <= n < r).  The threshold is
+ * other rows hold, and it cannot be selected.  Its estimate is left in the workspace as the
+ * marker -((32 g + n) * 2^-149): n the rows it examined (f <= n < r), g how many of those
+ * cells were read from the table (where the classes of the first f rows' cells fit in shared
+ * memory, f * c / 4 bytes <= 192 KiB, those cells are classified there and not read: g = n - f;
+ * otherwise g = n).  The threshold is
  * taken by the same call before the main pass, from the full estimate of a fixed sample (the
  * first four coordinates of every 256): the level-1 bin edge below a rank of the sample chosen
  * so that the threshold lies under the k-th largest |est| except with negligible probability.
@@ -200,8 +203,8 @@ gs_status gs_query_heavymix_workspace_size(int64_t d, int64_t k, size_t* bytes);
  * With est_out NULL, d >= 2^22, r >= 3 and c a power of two, rows are skipped as in
  * gs_query_topk with t = sqrt(l2sq / k) (rounded down to a bin edge): a coordinate that stops
  * has est^2 below the threshold, so it can only enter through the fill, and its estimate is
- * left in the workspace as -(n * 2^-149), n the rows it read; idx_out is the same as without
- * skipping. */
+ * left in the workspace as the marker -((32 n + n) * 2^-149), n the rows it read; idx_out is
+ * the same as without skipping. */
 gs_status gs_query_heavymix(const gs_sketch* sketch, int64_t d, int64_t k, uint64_t fill_seed,
                             int64_t* idx_out, float* est_out, double* l2sq_out, void* workspace,
                             size_t workspace_bytes, gs_stream stream);
