@@ -407,10 +407,12 @@ constexpr uint32_t kBitsBytes = 192u << 10;   // dynamic shared memory for the c
 
 constexpr int kBitsBlock = 1024;              // one CTA of 32 warps per SM
 
+// The class as two bits: bit 1 set when the cell counts below t (T < t), bit 0 when it counts
+// above -t (T > -t): 3 for |T| < t, 1 for T >= t, 2 for T <= -t, 0 for NaN.
 __device__ __forceinline__ uint32_t cell_class(float v, uint32_t pk) {
   const uint32_t b = __float_as_uint(v), key = b & 0x7FFFFFFFu;
-  if (key > 0x7F800000u) return 3u;
-  if (key < pk) return 0u;
+  if (key > 0x7F800000u) return 0u;
+  if (key < pk) return 3u;
   return (b >> 31) ? 2u : 1u;
 }
 
@@ -462,11 +464,7 @@ __global__ void __launch_bounds__(kBitsBlock, 1) k_query_bits(const __grid_const
       uint32_t cell[4][kF];  // bucket of each of the first kF rows, sign bit of the cell in bit 31
       int lt[4], gt[4], rows[4];
       bool done[4];
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        lt[t] = 0;
-        gt[t] = 0;
-      }
+      uint32_t count[4] = {0u, 0u, 0u, 0u};
       // the first kF rows: classes from shared memory, no table reads
 #pragma unroll
       for (int j = 0; j < kF; ++j) {
@@ -478,10 +476,12 @@ __global__ void __launch_bounds__(kBitsBlock, 1) k_query_bits(const __grid_const
           if (t < tmax) {
             const uint32_t b = (uint32_t)x & prm.cmask;
             const uint32_t g = (uint32_t)j * prm.c + b;
-            uint32_t cls = (sbits[g >> 4] >> ((g & 15u) * 2u)) & 3u;
-            if ((uint32_t)y & 1u) cls = (cls == 1u || cls == 2u) ? (3u - cls) : cls;
-            lt[t] += (cls == 0u || cls == 2u) ? 1 : 0;
-            gt[t] += (cls == 0u || cls == 1u) ? 1 : 0;
+            const uint32_t cls = (sbits[g >> 4] >> ((g & 15u) * 2u)) & 3u;
+            // a negative sign swaps the two bits; count[t] holds below-t in bits 0-7 and
+            // above-(-t) in bits 8-15: (cls * 0x201) >> 1 puts bit 1 at 0 and bit 0 at 8,
+            // cls * 0x81 puts bit 0 at 0 and bit 1 at 8
+            const uint32_t s = (uint32_t)y & 1u;
+            count[t] += ((cls * (s ? 0x81u : 0x201u)) >> (1u - s)) & 0x101u;
             cell[t][j] = b | signbit_of(y);
             x = step61_nb(x, prm.h.a[j]);
             y = step61_nb(y, prm.h.a2[j]);
@@ -490,6 +490,8 @@ __global__ void __launch_bounds__(kBitsBlock, 1) k_query_bits(const __grid_const
       }
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
+        lt[t] = (int)(count[t] & 0xFFu);
+        gt[t] = (int)(count[t] >> 8);
         rows[t] = kF;
         done[t] = pk != 0u && lt[t] >= kF && gt[t] >= kF;
       }
