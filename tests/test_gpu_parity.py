@@ -449,14 +449,17 @@ def _settle_threshold(v, f):
     return np.maximum(srt[f - 1], -srt[v.shape[0] - f])
 
 
-@pytest.mark.parametrize("r", [3, 4, 5, 7, 16])
-def test_pruned_rows_follow_the_rule(gs, H, r):
-    """The rows each coordinate read, from its marker, against the rule, with the signed cells
+@pytest.mark.parametrize("r,c", [(3, 1 << 16), (4, 1 << 16), (5, 1 << 16), (7, 1 << 16), (16, 1 << 16),
+                                 (5, 1 << 19), (7, 1 << 18)])
+def test_pruned_rows_follow_the_rule(gs, H, r, c):
+    """The rows each coordinate examined, from its marker, against the rule, with the signed cells
     recomputed on the host from the merged table and the hash values: one prune key t must
     exist such that every coordinate that stopped after n rows was settled by its first n cells
     (t above their settle threshold) and unsettled by its first n - 1 when n > r/2 + 1, and
-    every coordinate that read all r rows was unsettled by its first r - 1."""
-    d, c, k, seed = 4_200_007, 1 << 16, 4000, 60 + r
+    every coordinate that examined all r rows was unsettled by its first r - 1.  The cells read
+    are those the header states: all n examined ones, or, where the classes of the first
+    f = r/2 + 1 rows fit in 192 KiB of shared memory (the first five cases), n - f."""
+    d, k, seed = 4_200_007, 4000, 60 + r
     f = r // 2 + 1
     rng = np.random.default_rng(seed)
     sk = gs.gs_sketch_create(r, c, seed, 1, 0)
@@ -469,6 +472,8 @@ def test_pruned_rows_follow_the_rule(gs, H, r):
         torch.cuda.synchronize()
         e_int = H.host(ws[: 4 * d].view(torch.float32)).copy()
         pruned, n = H.pruned_rows(e_int, r)
+        g = ((e_int.view(np.uint32)[pruned] >> np.uint32(5)) & np.uint32(31)).astype(np.int64)
+        assert np.array_equal(g, n - f if f * c // 4 <= 192 << 10 else n), "cells read differ from the header"
         # markers name f <= n < r rows, so for r = 4 every one names 3
         assert pruned.mean() > 0.5 and (r - 1 == f or np.any(n > f)), "coordinates should stop at several row counts"
         T = np.empty(r * c, np.float32)
