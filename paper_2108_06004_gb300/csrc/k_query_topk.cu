@@ -396,8 +396,9 @@ __global__ void __launch_bounds__(kBlock, R <= 7 ? 4 : 1) k_query(const __grid_c
 
 // ---- the pruning query with the first rows classified in shared memory ---------------------
 // The settle rule needs, for each of the first f = r/2 + 1 cells of a coordinate, only which side
-// of the prune key t its value lies on.  For a row that is a class per table cell: 0 (|T| < t),
-// 1 (T >= t), 2 (T <= -t) or 3 (NaN); the sign hash of the coordinate swaps classes 1 and 2.
+// of the prune key t its value lies on.  For a row that is a class per table cell, two bits:
+// whether T counts below t and whether it counts above -t (3 for |T| < t, 1 for T >= t, 2 for
+// T <= -t, 0 for NaN); the sign hash of the coordinate swaps the two bits.
 // Where the classes of the first f rows fit in shared memory (2 bits per cell), k_pbits writes
 // them once per query and k_query_bits looks them up instead of reading those cells from L2.  A
 // coordinate that settles within the first f rows then reads no cell at all; one that examines
