@@ -1,4 +1,5 @@
-"""The row-skipping rule of the median query, checked on the host by brute force (no GPU).
+"""The row-skipping rule of the median query and the integer shortcuts of its kernels, checked
+on the host (no GPU).
 
 The query stops reading a coordinate's rows once, with f = r/2 + 1, at least f of the signed
 cells read so far are < t and at least f are > -t.  The claim that makes this safe: then the
@@ -70,3 +71,78 @@ def test_unsettled_rows_can_reach_the_threshold():
     read = np.array([0.1, -0.2, 2.0], np.float32)
     assert not settled(read, t, f)
     assert median_fp32(np.concatenate([read, np.array([2.0, 2.0], np.float32)])) >= t
+
+
+# ---- the query's integer shortcuts, checked against their definitions ----------------------
+
+P61 = (1 << 61) - 1
+M64 = (1 << 64) - 1
+
+
+def _reduce61(s):
+    """The query's compare-free reduction, in 64-bit wrap-around arithmetic."""
+    return ((s + (((s + 1) & M64) >> 61)) & M64) & P61
+
+
+def _fold61(x):
+    return (x & P61) + (x >> 61)
+
+
+def _affine61_nb(a, b, i):
+    p0 = (a & 0xFFFFFFFF) * i
+    p1 = (a >> 32) * i
+    s = (p1 >> 29) + ((p1 & ((1 << 29) - 1)) << 32) + _fold61(p0) + b
+    assert s < 3 << 61
+    return _reduce61(_fold61(s))
+
+
+def test_compare_free_modular_steps():
+    """For s < 2p, (s + ((s + 1) >> 61)) & p is s mod p; the affine evaluation built on it equals
+    (a i + b) mod p for a, b < p and i < 2^32, at the extremes and on random values."""
+    rng = np.random.default_rng(61)
+    edges = [0, 1, 2, P61 - 2, P61 - 1, 1 << 60, (1 << 60) - 1, (1 << 32) - 1, 1 << 32]
+    for x in edges:
+        for a in edges:
+            assert _reduce61(x + a) == (x + a) % P61
+    for _ in range(20000):
+        x, a = int(rng.integers(0, P61)), int(rng.integers(0, P61))
+        assert _reduce61(x + a) == (x + a) % P61
+    for a in [1, 2, P61 - 1, P61 - 2, (1 << 32) - 1, 1 << 32, (1 << 60) + 12345]:
+        for b in [0, 1, P61 - 1]:
+            for i in [0, 1, (1 << 31) - 1, 1 << 31, (1 << 32) - 1]:
+                assert _affine61_nb(a, b, i) == (a * i + b) % P61
+    for _ in range(20000):
+        a, b, i = int(rng.integers(1, P61)), int(rng.integers(0, P61)), int(rng.integers(0, 1 << 32))
+        assert _affine61_nb(a, b, i) == (a * i + b) % P61
+
+
+def _cell_class(T, pk):
+    bits = int(np.float32(T).view(np.uint32))
+    key = bits & 0x7FFFFFFF
+    if key > 0x7F800000:
+        return 0
+    if key < pk:
+        return 3
+    return 2 if bits >> 31 else 1
+
+
+def _tally(v, pk):
+    bits = int(np.float32(v).view(np.uint32))
+    key = bits & 0x7FFFFFFF
+    inside, number = key < pk, key <= 0x7F800000
+    return int(inside or (number and bits >> 31 == 1)), int(inside or (number and bits >> 31 == 0))
+
+
+def test_class_bits_count_like_the_values():
+    """A cell's two class bits, swapped by a negative sign and added into a packed pair of
+    counters by one multiply, count below t and above -t exactly as the signed value does."""
+    pk = int(np.float32(1.0).view(np.uint32)) & 0x7FFFFFFF
+    values = [0.0, -0.0, 0.5, -0.5, 1.0, -1.0, 2.0, -2.0, np.inf, -np.inf, 1e-30, -1e-30,
+              np.float32(1.0) * (1 - 2.0**-24), -np.float32(1.0) * (1 - 2.0**-24)]
+    nans = [np.uint32(0x7FC00000).view(np.float32), np.uint32(0xFFC00000).view(np.float32)]
+    for T in values + nans:
+        for s in (0, 1):
+            v = np.float32(T) if s == 0 else np.uint32(int(np.float32(T).view(np.uint32)) ^ 0x80000000).view(np.float32)
+            c = _cell_class(T, pk)
+            packed = ((c * (0x81 if s else 0x201)) >> (1 - s)) & 0x101
+            assert (packed & 0xFF, packed >> 8) == _tally(v, pk), (T, s)
