@@ -406,6 +406,33 @@ def test_pruned_query_matches_full_query(gs, H, r, adversarial):
         gs.gs_sketch_destroy(sk)
 
 
+@pytest.mark.parametrize("k,r,c", [(1, 5, 1 << 16), (7, 5, 1 << 16), (1_400_002, 5, 1 << 16), (1, 7, 1 << 18),
+                                   (1_400_002, 7, 1 << 18)])
+def test_pruned_query_extreme_k(gs, H, k, r, c):
+    """Pruning queries at the extremes of k (one coordinate; a third of them), on the kernel that
+    classifies the first rows in shared memory (c = 2^16) and on the one that reads them
+    (r = 7, c = 2^18): the selection equals the full query's, every selected estimate is exact,
+    and every marker lies below the k-th largest |est|."""
+    d, seed = 4_200_007, 70 + k % 97 + r
+    rng = np.random.default_rng(seed)
+    sk = gs.gs_sketch_create(r, c, seed, 1, 0)
+    try:
+        ws = torch.empty(gs.gs_query_topk_workspace_size(d, k), dtype=torch.uint8, device="cuda")
+        idx = torch.empty(k, dtype=torch.int64, device="cuda")
+        idx_full = torch.empty(k, dtype=torch.int64, device="cuda")
+        est_full = torch.empty(d, dtype=torch.float32, device="cuda")
+        gs.gs_sketch_insert(sk, 0, _dev(_prune_input(rng, d, min(k, 4000), False)), d)
+        gs.gs_sketch_merge_tree(sk, 1)
+        gs.gs_query_topk(sk, d, k, idx, None, ws)
+        torch.cuda.synchronize()
+        got, e_int = H.host(idx).copy(), H.host(ws[: 4 * d].view(torch.float32)).copy()
+        gs.gs_query_topk(sk, d, k, idx_full, est_full, ws)
+        torch.cuda.synchronize()
+        _check_pruned_against_full(H, got, e_int, H.host(idx_full), H.host(est_full), k, r)
+    finally:
+        gs.gs_sketch_destroy(sk)
+
+
 def test_pruned_queries_on_two_streams(gs, H):
     """Queries of one sketch on two streams at once, each with its own workspace, one on natural
     and one on adversarial data (a second sketch), interleaved launch after launch: a query keeps
